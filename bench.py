@@ -1,0 +1,431 @@
+#!/usr/bin/env python
+"""Benchmark of the GPU-resident LLM prefix (blocks [0, k) of a 7B-class backbone).
+
+One step = one frame through the prefix: a 2304-token prefill of blocks [0, 16) (all
+projections, attention and KV writes on the tensor-core path) and the boundary hand-off of
+h^(16) [2304, 4096] bf16 to pinned host memory on a side stream, overlapped with the next
+frame's prefill (the GPU side of the cross-frame pipeline, Sec. IV-C). A decode phase then
+times 64 single-token steps of the same 16 blocks against a 2304-position context.
+
+Inputs are seeded synthetic tensors of the workload's shapes (the paper's Bench2Drive frames
+and Orion weights are not available): weights ~ N(0, 0.02), hidden states ~ N(0, 1).
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun each rank runs an independent replica (the prefix has no exchange step on one
+GPU); the slowest rank's time is reported and ``value`` counts all ranks' tokens.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "prefix prefill tokens/s & % bf16 TC peak; decode µs/step & HBM GB/s (1 GB300)"
+WORKLOAD = "7b_prefix16_2304tok"
+DECODE_WORKLOAD = "7b_decode16_ctx2304"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d["bf16_tflops_sustained"], "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------------------------------------
+# distributed plumbing (replicas; only the barrier and the max-reduce of the time cross ranks)
+# ------------------------------------------------------------------------------------------
+class Dist:
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+
+    def init(self, backend: str):
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float, device=None) -> float:
+        if not self.pg:
+            return x
+        import torch
+        t = torch.tensor([x], dtype=torch.float64, device=device)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+# ------------------------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ------------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict | None:
+        if not self.proc:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax = max(smax, float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------
+# CPU oracle timing (baseline and reference arm): only here and in the tests is oracle/ run
+# ------------------------------------------------------------------------------------------
+_ORACLE_W = {}
+
+
+def oracle_prefill_time(n_tokens: int, seed: int = 0) -> tuple[float, int]:
+    """Seconds for the float64 oracle to run one 7B-class block over the first ``n_tokens``
+    tokens of the workload's frame (weights converted outside the timed region)."""
+    import oracle
+    wl = synth.WORKLOADS[WORKLOAD]
+    s = wl.shape
+    if seed not in _ORACLE_W:
+        _ORACLE_W[seed] = oracle.LayerWeights.from_bf16(synth.layer_weights(s, seed, 0))
+    w = _ORACLE_W[seed]
+    x = oracle.bf16_to_f64(synth.hidden_states(n_tokens, s.hidden, seed, min(n_tokens, wl.visual_tokens),
+                                               wl.visual_scale))
+    cache = oracle.KVCache([0], s.n_kv_heads, s.head_dim, n_tokens)
+    t0 = time.perf_counter()
+    oracle.block_forward(x, w, cache, 0, s)
+    return time.perf_counter() - t0, os.cpu_count() or 1
+
+
+def cpu_threads() -> int:
+    for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(v, "").isdigit():
+            return int(os.environ[v])
+    return os.cpu_count() or 1
+
+
+def run_reference(args, dist: Dist):
+    """The oracle as it stands, timed on the host cores (rank 0 only)."""
+    if dist.rank != 0:
+        return
+    wl = synth.WORKLOADS[WORKLOAD]
+    sample_tokens = 512
+    for _ in range(args.warmup):
+        oracle_prefill_time(sample_tokens)
+    t = 0.0
+    for _ in range(args.steps):
+        dt, _ = oracle_prefill_time(sample_tokens)
+        t += dt
+    per_step = t / args.steps
+    # one step of the workload = 16 blocks; the sample is 1 block over the first 512 tokens
+    tok_s = sample_tokens / (per_step * wl.prefix_layers)
+    sample = (f"1 of {wl.prefix_layers} blocks over the first {sample_tokens} of {wl.n_tokens} tokens per step, "
+              f"extrapolated x{wl.prefix_layers} blocks (float64 numpy oracle)")
+    line = {"impl": "reference", "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * wl.prefix_layers * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "blocks": wl.prefix_layers, "tokens": wl.n_tokens, "hidden": 4096},
+            "cpu_baseline": {"value": tok_s, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": tok_s, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------------
+# GPU arm
+# ------------------------------------------------------------------------------------------
+def to_dev(bits, torch):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def run_ours(args, dist: Dist):
+    import torch
+
+    import paper_2608_14586_gb300 as vla
+    torch.cuda.set_device(dist.local)
+    dist.init("nccl")
+    vla.build()
+    vla.load()
+    hbm_peak, bf16_burst, bf16_sust, peak_src = _peaks()
+    wl = synth.WORKLOADS[WORKLOAD]
+    dwl = synth.WORKLOADS[DECODE_WORKLOAD]
+    s = wl.shape
+    L = wl.prefix_layers
+    M = wl.n_tokens
+    D = s.hidden
+    dec_steps = dwl.decode_steps
+    max_ctx = max(M, dwl.prefill_ctx + dec_steps + 8)
+    seed = wl.seed
+
+    # ---- model: the 16 prefix blocks (seeded synthetic weights), library-owned copies
+    layers = []
+    for l in range(L):
+        layers.append({k: to_dev(v, torch) for k, v in synth.layer_weights(s, seed, l).items()})
+    cfg = vla.VlaConfig(hidden=D, n_heads=s.n_heads, n_kv_heads=s.n_kv_heads, head_dim=s.head_dim, ffn=s.ffn,
+                        rms_eps=s.rms_eps, rope_base=s.rope_base, max_ctx=max_ctx)
+    p = vla.vla_prefix_create(cfg, layers)
+    del layers
+    torch.cuda.empty_cache()
+    kv = vla.vla_kv_create(p, 0, L, max_ctx)
+
+    xb = synth.hidden_states(M, D, seed, wl.visual_tokens, wl.visual_scale)
+    x = to_dev(xb, torch)
+    outs = [torch.empty((M, D), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    pinned = [torch.empty((M, D), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    main = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    ready = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    for e in done:
+        e.record(side)
+    launches = [0]
+
+    def step(i: int, x_in):
+        b = i & 1
+        main.wait_event(done[b])                   # frame i-2's copy of this buffer has landed
+        vla.vla_kv_reset(kv, main)                  # a new frame starts at position 0
+        vla.vla_prefix_prefill(p, x_in, M, 0, L, kv, outs[b], main)
+        launches[0] += vla.vla_last_launch_count(p) + 1
+        ready[b].record(main)
+        vla.vla_boundary_to_host(outs[b], M, D, pinned[b], side, ready[b], done[b])
+
+    for i in range(args.warmup):
+        step(i, x)
+    torch.cuda.synchronize()
+    vla.vla_prefix_stage_times(p)  # discard
+
+    gpu_id = os.environ.get("CUDA_VISIBLE_DEVICES", str(dist.local)).split(",")[0] \
+        if dist.world == 1 else str(dist.local)
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    dist.barrier()
+    torch.cuda.synchronize()
+    launches[0] = 0
+    vla.vla_prefix_set_timing(p, True)
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(main)
+    for i in range(args.steps):
+        step(i, x)
+    main.wait_event(done[(args.steps - 1) & 1])
+    t_end.record(main)
+    torch.cuda.synchronize()
+    vla.vla_prefix_set_timing(p, False)
+    dist.barrier()
+    ms = t_start.elapsed_time(t_end) / args.steps
+    ms = dist.max(ms, "cuda")
+    stages = vla.vla_prefix_stage_times(p)
+    prefill_launches = launches[0]
+    assert vla.vla_last_async_error(p) == 0
+
+    # roofline of the dominant kernel: gate/up projection + SwiGLU (51% of the GEMM flops)
+    gu_ms, gu_n = stages["gemm_gateup"]
+    gu_flops = 2.0 * M * (2 * s.ffn) * D
+    gu_tflops = gu_flops / (gu_ms / gu_n * 1e-3) / 1e12 if gu_n else 0.0
+    block_flops = 2.0 * M * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                             D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * M * M * s.head_dim * s.n_heads
+    step_tflops = block_flops * L / (ms * 1e-3) / 1e12
+
+    # ---- end to end through the C ABI with host buffers (H2D of the frame, D2H of h^(16))
+    host_in = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).pin_memory()
+    x_dev = torch.empty_like(x)
+
+    def e2e_step(i):
+        b = i & 1
+        main.wait_event(done[b])
+        x_dev.copy_(host_in, non_blocking=True)
+        vla.vla_kv_reset(kv, main)
+        vla.vla_prefix_prefill(p, x_dev, M, 0, L, kv, outs[b], main)
+        ready[b].record(main)
+        vla.vla_boundary_to_host(outs[b], M, D, pinned[b], side, ready[b], done[b])
+
+    for i in range(args.warmup):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        e2e_step(i)
+    done[(args.steps - 1) & 1].synchronize()
+    torch.cuda.synchronize()
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / args.steps
+    e2e_ms = dist.max(e2e_ms, "cuda")
+    # the boundary that reached the host equals the device result
+    assert torch.equal(pinned[(args.steps - 1) & 1].view(torch.int16).cpu(),
+                       outs[(args.steps - 1) & 1].view(torch.int16).cpu())
+
+    # ---- decode: 64 single-token steps against a 2304-position random context
+    ctx0 = dwl.prefill_ctx
+    for l in range(L):
+        kb, vb = synth.random_kv(ctx0, s, dwl.seed, l)
+        kp, vp = vla.vla_kv_data(kv, l)
+        for ptr, bits in ((kp, kb), (vp, vb)):
+            src = to_dev(bits, torch)  # [Hkv, ctx0, dh] -> rows of the [Hkv, max_ctx, dh] plane
+            for g in range(s.n_kv_heads):
+                dst = _dev_view(ptr + g * max_ctx * s.head_dim * 2, ctx0 * s.head_dim, torch)
+                dst.copy_(src[g].reshape(-1))
+    torch.cuda.synchronize()
+    xd = to_dev(np.stack([synth.decode_hidden(t, D, dwl.seed)[0] for t in range(dec_steps)]), torch)
+    yd = torch.empty((1, D), dtype=torch.bfloat16, device="cuda")
+
+    def decode_run():
+        vla.vla_kv_set_length(kv, ctx0, main)
+        n = 1
+        for t in range(dec_steps):
+            vla.vla_prefix_decode(p, xd[t:t + 1], 0, L, kv, yd, main)
+            n += vla.vla_last_launch_count(p)
+        return n
+
+    for _ in range(max(1, args.warmup // 2)):
+        decode_run()
+    torch.cuda.synchronize()
+    dist.barrier()
+    vla.vla_prefix_stage_times(p)
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(main)
+    reps = max(1, args.steps // 8)
+    dec_launches = 0
+    for _ in range(reps):
+        dec_launches += decode_run()
+    d1.record(main)
+    torch.cuda.synchronize()
+    clock_info = clocks.stop()
+    dist.barrier()
+    dec_us = d0.elapsed_time(d1) * 1e3 / (reps * dec_steps)
+    dec_us = dist.max(dec_us, "cuda")
+    assert vla.vla_last_async_error(p) == 0
+    weight_bytes = L * 2 * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                            D * s.n_heads * s.head_dim + 3 * s.ffn * D)
+    avg_ctx = ctx0 + (dec_steps + 1) / 2
+    kv_bytes = L * 2 * s.n_kv_heads * s.head_dim * 2 * avg_ctx
+    dec_bytes = weight_bytes + kv_bytes
+    dec_gbs = dec_bytes / (dec_us * 1e-6) / 1e9
+
+    # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame
+    cpu = None
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        t_cpu, _ = oracle_prefill_time(M)
+        cpu = {"value": M / (t_cpu * L), "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
+               "sample": f"1 of {L} blocks over the full {M}-token frame ({t_cpu:.1f} s), extrapolated x{L} "
+                         f"blocks; float64 numpy oracle"}
+
+    if dist.rank == 0:
+        tok_s = M * dist.world / (ms * 1e-3)
+        line = {
+            "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": dist.world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "blocks": L, "tokens": M, "hidden": D,
+                       "heads": f"{s.n_heads}q/{s.n_kv_heads}kv x {s.head_dim}", "ffn": s.ffn,
+                       "boundary_bytes": M * D * 2, "l2": "weights 5.67 GB streamed per step > 129 MB L2",
+                       "parallelism": f"replicas x{dist.world}"},
+            "roofline": {"kernel": "gemm_gateup (tcgen05, SwiGLU epilogue)", "bound": "tensor",
+                         "achieved": gu_tflops, "peak": bf16_sust, "unit": "TFLOP/s", "frac": gu_tflops / bf16_sust,
+                         "peak_source": f"{peak_src} bf16 sustained", "traffic": None,
+                         "flops_per_launch": gu_flops, "avg_launch_ms": gu_ms / max(gu_n, 1)},
+            "step_tflops": step_tflops, "step_frac_of_peak": step_tflops / bf16_sust,
+            "cpu_baseline": cpu,
+            "e2e": {"value": M * dist.world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
+                    "h2d_bytes_per_step": M * D * 2, "d2h_bytes_per_step": M * D * 2},
+            "gpu_launches": prefill_launches,
+            "clocks": clock_info,
+            "stages_ms_per_launch": {k: round(v[0] / v[1], 4) for k, v in stages.items() if v[1]},
+            "decode": {"workload": DECODE_WORKLOAD, "us_per_step": dec_us, "bytes_per_step": dec_bytes,
+                       "hbm_gbs": dec_gbs, "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm_peak,
+                                                        "unit": "GB/s", "frac": dec_gbs / hbm_peak,
+                                                        "peak_source": f"{peak_src} copy bandwidth",
+                                                        "traffic": None},
+                       "gpu_launches_per_step": dec_launches / (reps * dec_steps)},
+        }
+        print(json.dumps(line), flush=True)
+    vla.vla_kv_destroy(kv)
+    vla.vla_prefix_destroy(p)
+    dist.close()
+
+
+class _CudaArray:
+    def __init__(self, ptr: int, numel: int):
+        self.__cuda_array_interface__ = {"data": (int(ptr), False), "shape": (int(numel),), "typestr": "<i2",
+                                         "strides": None, "version": 3}
+
+
+def _dev_view(ptr, numel, torch):
+    return torch.as_tensor(_CudaArray(ptr, numel), device="cuda").view(torch.bfloat16)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    dist = Dist()
+    if args.impl == "reference":
+        run_reference(args, dist)
+    else:
+        run_ours(args, dist)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,238 @@
+"""GB300 LLM-prefix library: Python binding of the C ABI in ``include/vla_prefix.h``.
+
+Argument marshalling only: every stage of the prefix forward runs in the CUDA kernels of
+``libvla_prefix.so`` (built in-tree from ``csrc/`` by ``build()``). Tensors are passed as
+device pointers (torch tensors are accepted for convenience: their ``data_ptr()`` is used),
+streams as ``torch.cuda.Stream`` or raw ``cudaStream_t`` integers. There is no CPU fallback:
+``load()`` raises if the library has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from ._build import LIB as LIB_PATH
+from ._build import build as _build_lib
+
+__all__ = [
+    "build", "load", "VlaError", "VlaConfig", "VlaLayerWeights",
+    "vla_prefix_create", "vla_prefix_destroy", "vla_kv_create", "vla_kv_destroy", "vla_kv_reset",
+    "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_set_length", "vla_prefix_prefill",
+    "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
+    "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
+    "vla_prefix_stage_times", "STATUS", "STAGES",
+]
+
+# stage ids of vla_prefix_stage_times (VLA_STAGE_* in vla_prefix.h)
+STAGES = ("rowstat", "gemm_qkv", "attn_prefill", "gemm_o", "gemm_gateup", "gemm_down", "kv_len",
+          "dec_qkv", "dec_attn", "dec_combine", "dec_o", "dec_gateup", "dec_down")
+
+STATUS = {0: "VLA_OK", 1: "VLA_ERR_INVALID_ARG", 2: "VLA_ERR_SHAPE", 3: "VLA_ERR_RANGE", 4: "VLA_ERR_KV_FULL",
+          5: "VLA_ERR_NOT_PINNED", 6: "VLA_ERR_OOM", 7: "VLA_ERR_CUDA", 8: "VLA_ERR_TIMEOUT",
+          9: "VLA_ERR_UNSUPPORTED"}
+
+
+class VlaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        self.name = STATUS.get(status, str(status))
+        super().__init__(f"{where}: {self.name} ({_lib.vla_status_str(status).decode() if _lib else status})")
+
+
+class VlaConfig(ctypes.Structure):
+    _fields_ = [("hidden", ctypes.c_int), ("n_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("ffn", ctypes.c_int), ("rms_eps", ctypes.c_float),
+                ("rope_base", ctypes.c_float), ("max_ctx", ctypes.c_int)]
+
+
+_WNAMES = ("w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down", "g_attn", "g_mlp")
+
+
+class VlaLayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in _WNAMES]
+
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the CUDA library (nvcc, sm_103a) in-tree; returns its path."""
+    return _build_lib(force=force)
+
+
+def load():
+    """Load ``libvla_prefix.so``; raises if it has not been built (no fallback exists)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: run paper_2608_14586_gb300.build() (needs nvcc)")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, V = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p
+    sig = {
+        "vla_prefix_create": ([ctypes.POINTER(VlaConfig), ctypes.POINTER(VlaLayerWeights), I,
+                               ctypes.POINTER(P)], I),
+        "vla_prefix_destroy": ([P], I),
+        "vla_kv_create": ([P, I, I, I, ctypes.POINTER(P)], I),
+        "vla_kv_destroy": ([P], I),
+        "vla_kv_reset": ([P, V], I),
+        "vla_kv_length": ([P], I),
+        "vla_kv_layer_length": ([P, I], I),
+        "vla_kv_data": ([P, I, ctypes.POINTER(P), ctypes.POINTER(P)], I),
+        "vla_kv_set_length": ([P, I, V], I),
+        "vla_prefix_prefill": ([P, V, I, I, I, P, V, V], I),
+        "vla_prefix_decode": ([P, V, I, I, P, V, V], I),
+        "vla_boundary_to_host": ([V, I, I, V, V, V, V], I),
+        "vla_last_async_error": ([P], I),
+        "vla_status_str": ([I], ctypes.c_char_p),
+        "vla_last_launch_count": ([P], I),
+        "vla_op_gemm_bf16": ([V, V, I, I, I, V, V], I),
+        "vla_op_attention_prefill": ([V, V, V, I, I, I, I, I, I, V, V], I),
+        "vla_prefix_set_timing": ([P, I], I),
+        "vla_prefix_stage_times": ([P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int), I], I),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = lib
+    return lib
+
+
+def _ptr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    if hasattr(x, "value"):
+        return x.value
+    raise TypeError(f"cannot take a device pointer of {type(x)}")
+
+
+def _stream(s) -> int | None:
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    if hasattr(s, "cuda_stream"):
+        return s.cuda_stream
+    raise TypeError(f"not a stream: {type(s)}")
+
+
+def _event(e) -> int | None:
+    if e is None:
+        return None
+    if isinstance(e, int):
+        return e
+    if hasattr(e, "cuda_event"):
+        return e.cuda_event
+    raise TypeError(f"not an event: {type(e)}")
+
+
+def _check(st: int, where: str):
+    if st != 0:
+        raise VlaError(st, where)
+
+
+def vla_status_str(status: int) -> str:
+    return load().vla_status_str(status).decode()
+
+
+def vla_prefix_create(cfg: VlaConfig, layers) -> ctypes.c_void_p:
+    """``layers``: sequence of mappings name -> device tensor / pointer (see VlaLayerWeights)."""
+    lib = load()
+    arr = (VlaLayerWeights * len(layers))()
+    for i, w in enumerate(layers):
+        for n in _WNAMES:
+            setattr(arr[i], n, _ptr(w[n]))
+    out = ctypes.c_void_p()
+    _check(lib.vla_prefix_create(ctypes.byref(cfg), arr, len(layers), ctypes.byref(out)), "vla_prefix_create")
+    return out
+
+
+def vla_prefix_destroy(p):
+    _check(load().vla_prefix_destroy(p), "vla_prefix_destroy")
+
+
+def vla_kv_create(p, layer_begin: int, layer_end: int, max_ctx: int) -> ctypes.c_void_p:
+    out = ctypes.c_void_p()
+    _check(load().vla_kv_create(p, layer_begin, layer_end, max_ctx, ctypes.byref(out)), "vla_kv_create")
+    return out
+
+
+def vla_kv_destroy(kv):
+    _check(load().vla_kv_destroy(kv), "vla_kv_destroy")
+
+
+def vla_kv_reset(kv, stream=None):
+    _check(load().vla_kv_reset(kv, _stream(stream)), "vla_kv_reset")
+
+
+def vla_kv_length(kv) -> int:
+    return load().vla_kv_length(kv)
+
+
+def vla_kv_layer_length(kv, layer: int) -> int:
+    return load().vla_kv_layer_length(kv, layer)
+
+
+def vla_kv_data(kv, layer: int):
+    k, v = ctypes.c_void_p(), ctypes.c_void_p()
+    _check(load().vla_kv_data(kv, layer, ctypes.byref(k), ctypes.byref(v)), "vla_kv_data")
+    return k.value, v.value
+
+
+def vla_kv_set_length(kv, length: int, stream=None):
+    _check(load().vla_kv_set_length(kv, length, _stream(stream)), "vla_kv_set_length")
+
+
+def vla_prefix_prefill(p, hidden_in, n_tokens: int, layer_begin: int, layer_end: int, kv, hidden_out,
+                       stream=None):
+    _check(load().vla_prefix_prefill(p, _ptr(hidden_in), n_tokens, layer_begin, layer_end, kv, _ptr(hidden_out),
+                                     _stream(stream)), "vla_prefix_prefill")
+
+
+def vla_prefix_decode(p, hidden_in, layer_begin: int, layer_end: int, kv, hidden_out, stream=None):
+    _check(load().vla_prefix_decode(p, _ptr(hidden_in), layer_begin, layer_end, kv, _ptr(hidden_out),
+                                    _stream(stream)), "vla_prefix_decode")
+
+
+def vla_boundary_to_host(hidden_out, n_tokens: int, hidden: int, pinned_dst, side_stream=None, ready=None,
+                         done=None):
+    _check(load().vla_boundary_to_host(_ptr(hidden_out), n_tokens, hidden, _ptr(pinned_dst), _stream(side_stream),
+                                       _event(ready), _event(done)), "vla_boundary_to_host")
+
+
+def vla_last_async_error(p) -> int:
+    return load().vla_last_async_error(p)
+
+
+def vla_last_launch_count(p) -> int:
+    return load().vla_last_launch_count(p)
+
+
+def vla_op_gemm_bf16(A, B, M: int, N: int, K: int, C, stream=None):
+    _check(load().vla_op_gemm_bf16(_ptr(A), _ptr(B), M, N, K, _ptr(C), _stream(stream)), "vla_op_gemm_bf16")
+
+
+def vla_op_attention_prefill(q, k_plane, v_plane, n_tokens: int, n_heads: int, n_kv_heads: int, head_dim: int,
+                             max_ctx: int, pos0: int, out, stream=None):
+    _check(load().vla_op_attention_prefill(_ptr(q), _ptr(k_plane), _ptr(v_plane), n_tokens, n_heads, n_kv_heads,
+                                           head_dim, max_ctx, pos0, _ptr(out), _stream(stream)),
+           "vla_op_attention_prefill")
+
+
+def vla_prefix_set_timing(p, enable: bool):
+    _check(load().vla_prefix_set_timing(p, 1 if enable else 0), "vla_prefix_set_timing")
+
+
+def vla_prefix_stage_times(p) -> dict:
+    """{stage name: (milliseconds, launches)} accumulated since the last read."""
+    n = len(STAGES)
+    ms = (ctypes.c_float * n)()
+    cnt = (ctypes.c_int * n)()
+    _check(load().vla_prefix_stage_times(p, ms, cnt, n), "vla_prefix_stage_times")
+    return {STAGES[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}

@@ -1,0 +1,123 @@
+// Small kernels around the GEMMs: RMSNorm row statistics, the rotary cos/sin table, weight
+// repacking at create time, and KV-length updates.
+#include "common.cuh"
+#include "internal.h"
+
+namespace vla {
+
+namespace {
+
+// One warp per row: rinv = 1 / sqrt(mean(x^2) + eps), fp32 sum of squares, 16-byte loads.
+__global__ void rowstat_kernel(const bf16* __restrict__ x, int M, int D, int ld, float eps,
+                               float* __restrict__ rinv) {
+    const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= M) return;
+    const bf16* xr = x + (size_t)row * ld;
+    float acc = 0.f;
+    for (int c = lane * 8; c < D; c += 32 * 8) {
+        const uint4 v = *reinterpret_cast<const uint4*>(xr + c);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float a = bf16_lo(w[i]), b = bf16_hi(w[i]);
+            acc = fmaf(a, a, acc);
+            acc = fmaf(b, b, acc);
+        }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) rinv[row] = 1.0f / sqrtf(acc / (float)D + eps);
+}
+
+// table[pos][j] = (cos, sin)(pos * base^(-2j/dh)), angles in float64
+__global__ void rope_table_kernel(float2* table, int max_ctx, int dh, double base) {
+    const int half = dh / 2;
+    const long long n = (long long)max_ctx * half;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const int pos = (int)(i / half), j = (int)(i % half);
+        const double theta = pow(base, -2.0 * (double)j / (double)dh);
+        const double ang = (double)pos * theta;
+        table[i] = make_float2((float)cos(ang), (float)sin(ang));
+    }
+}
+
+// Weight repack of one layer (see RepackDst in internal.h).
+__global__ void repack_kernel(RepackSrc s, RepackDst d, int D, int H, int Hkv, int dh, int F, int F_pad) {
+    const long long qn = (long long)H * dh, kvn = (long long)Hkv * dh;
+    const long long n_qkv = (qn + 2 * kvn) * D;
+    const long long n_o = (long long)D * H * dh;
+    const long long n_gu = 2LL * F_pad * D;
+    const long long n_d = (long long)D * F_pad;
+    const long long total = n_qkv + n_o + n_gu + n_d;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        long long j = i;
+        if (j < n_qkv) {
+            const long long r = j / D;
+            const int k = (int)(j % D);
+            const float gk = __bfloat162float(s.g_attn[k]);
+            float w;
+            if (r < qn) w = __bfloat162float(s.w_q[r * D + k]);
+            else if (r < qn + kvn) w = __bfloat162float(s.w_k[(r - qn) * D + k]);
+            else w = __bfloat162float(s.w_v[(r - qn - kvn) * D + k]);
+            d.w_qkv[j] = __float2bfloat16_rn(w * gk);
+            continue;
+        }
+        j -= n_qkv;
+        if (j < n_o) {
+            d.w_o[j] = s.w_o[j];
+            continue;
+        }
+        j -= n_o;
+        if (j < n_gu) {
+            const long long r = j / D;
+            const int k = (int)(j % D);
+            const long long grp = r / 256, w_in = r % 256;
+            const long long f = grp * 128 + (w_in < 128 ? w_in : w_in - 128);
+            float w = 0.f;
+            if (f < F) w = __bfloat162float(w_in < 128 ? s.w_gate[f * D + k] : s.w_up[f * D + k]);
+            d.w_gu[j] = __float2bfloat16_rn(w * __bfloat162float(s.g_mlp[k]));
+            continue;
+        }
+        j -= n_gu;
+        {
+            const long long r = j / F_pad;
+            const int k = (int)(j % F_pad);
+            d.w_d[j] = (k < F) ? s.w_down[r * F + k] : __float2bfloat16_rn(0.f);
+        }
+    }
+}
+
+__global__ void set_lengths_kernel(int* d_len, int count, int value) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < count) d_len[i] = value;
+}
+
+}  // namespace
+
+cudaError_t launch_rowstat(const bf16* x, int M, int D, int ld, float eps, float* rinv, cudaStream_t stream) {
+    if (M <= 0) return cudaSuccess;
+    const int rows_per_block = 8;
+    rowstat_kernel<<<(M + rows_per_block - 1) / rows_per_block, rows_per_block * 32, 0, stream>>>(x, M, D, ld, eps,
+                                                                                                  rinv);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream) {
+    rope_table_kernel<<<256, 256, 0, stream>>>(table, max_ctx, head_dim, base);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_repack(const RepackSrc& s, const RepackDst& d, int D, int H, int Hkv, int dh, int F, int F_pad,
+                          cudaStream_t stream) {
+    repack_kernel<<<1024, 256, 0, stream>>>(s, d, D, H, Hkv, dh, F, F_pad);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_set_lengths(int* d_len, int count, int value, cudaStream_t stream) {
+    if (count <= 0) return cudaSuccess;
+    set_lengths_kernel<<<(count + 127) / 128, 128, 0, stream>>>(d_len, count, value);
+    return cudaGetLastError();
+}
+
+}  // namespace vla

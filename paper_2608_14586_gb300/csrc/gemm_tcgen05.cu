@@ -1,0 +1,407 @@
+// Persistent warp-specialised bf16 GEMM on the 5th-generation tensor cores (tcgen05).
+//
+//   C[M, N] = A[M, K] * B[N, K]^T, fp32 accumulation in tensor memory (TMEM).
+//
+// Roles per CTA (192 threads, one CTA per SM):
+//   warp 0      one thread issues TMA tile loads (A: 128 x 64, B: BN x 64, 128-byte swizzle)
+//               into a STAGES-deep shared-memory ring guarded by full/empty mbarriers;
+//   warp 1      allocates 2*BN TMEM columns; one thread issues tcgen05.mma (M=128, N=BN,
+//               K=16) and commits each stage back to the producer and each finished tile to
+//               the epilogue;
+//   warps 2..5  epilogue: each warp reads its 32-lane quarter of the accumulator with
+//               tcgen05.ld, applies the fused step and stores bf16 results.
+// Two accumulator buffers let the epilogue of tile i overlap the mainloop of tile i+1.
+// Tiles are walked M-fastest so CTAs running together share the weight (B) tiles in L2.
+//
+// Fused epilogues (the block stages of the decoder, see the header of runtime.cu):
+//   kEpiQKV     RMSNorm row scale, rotate-half RoPE of q and k, q to the query buffer,
+//               post-RoPE k and v to the layer's KV cache at positions pos0 + row
+//   kEpiResid   residual add (attention output projection, MLP down projection)
+//   kEpiSwiGLU  RMSNorm row scale and silu(gate) * up on 128-column interleaved tiles
+#include "common.cuh"
+#include "internal.h"
+
+namespace vla {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+
+template <int BN>
+struct GemmCfg {
+    static constexpr int STAGES = (BN == 256) ? 4 : 6;
+    static constexpr uint32_t A_BYTES = kBM * kBK * 2;
+    static constexpr uint32_t B_BYTES = BN * kBK * 2;
+    static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr uint32_t TMEM_COLS = 2 * BN;
+    static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
+};
+
+VLA_DEV float f32(uint32_t u) { return __uint_as_float(u); }
+
+VLA_DEV void store_bf16x32(bf16* dst, const float (&v)[32]) {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        uint4 o;
+        o.x = pack_bf16x2(v[i * 8 + 0], v[i * 8 + 1]);
+        o.y = pack_bf16x2(v[i * 8 + 2], v[i * 8 + 3]);
+        o.z = pack_bf16x2(v[i * 8 + 4], v[i * 8 + 5]);
+        o.w = pack_bf16x2(v[i * 8 + 6], v[i * 8 + 7]);
+        d[i] = o;
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// Epilogues. Each thread owns one output row (TMEM lane); all 32 lanes of a warp execute
+// every tcgen05.ld; stores are masked per row / column.
+// ---------------------------------------------------------------------------------------
+template <int BN>
+VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& ep) {
+    const bool row_ok = row < ep.M;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        const int col = n0 + c;
+        if (!row_ok || col >= ep.N) continue;
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+        bf16* op = ep.out + (size_t)row * ep.ld_out + col;
+        if (col + 32 <= ep.N) {
+            if (ep.resid) {
+                const uint4* rp = reinterpret_cast<const uint4*>(ep.resid + (size_t)row * ep.ld_resid + col);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    uint4 q = rp[i];
+                    v[i * 8 + 0] += bf16_lo(q.x);
+                    v[i * 8 + 1] += bf16_hi(q.x);
+                    v[i * 8 + 2] += bf16_lo(q.y);
+                    v[i * 8 + 3] += bf16_hi(q.y);
+                    v[i * 8 + 4] += bf16_lo(q.z);
+                    v[i * 8 + 5] += bf16_hi(q.z);
+                    v[i * 8 + 6] += bf16_lo(q.w);
+                    v[i * 8 + 7] += bf16_hi(q.w);
+                }
+            }
+            store_bf16x32(op, v);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                if (col + i < ep.N) {
+                    float x = v[i];
+                    if (ep.resid) x += __bfloat162float(ep.resid[(size_t)row * ep.ld_resid + col + i]);
+                    op[i] = __float2bfloat16_rn(x);
+                }
+            }
+        }
+    }
+}
+
+template <int BN>
+VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
+    const bool row_ok = row < ep.M;
+    const float s = row_ok ? ep.rinv[row] : 0.f;
+    const int pos = ep.pos0 + row;
+    const int dh = ep.head_dim;
+    const int half = dh >> 1;
+    const int region = (n0 < ep.q_cols) ? 0 : ((n0 < ep.q_cols + ep.kv_cols) ? 1 : 2);
+    if (region == 2) {
+        // values: no rotation
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+            uint32_t r[32];
+            tmem_ld32(taddr + c, r);
+            if (!row_ok) continue;
+            const int n = n0 + c - ep.q_cols - ep.kv_cols;
+            const int g = n / dh, d = n % dh;
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = f32(r[i]) * s;
+            store_bf16x32(ep.vcache + ((size_t)g * ep.max_ctx + pos) * dh + d, v);
+        }
+        return;
+    }
+    const float2* rope = ep.rope + (size_t)(row_ok ? pos : 0) * half;
+#pragma unroll 1
+    for (int hb = 0; hb < BN; hb += dh) {
+#pragma unroll 1
+        for (int c = 0; c < half; c += 32) {
+            uint32_t ra[32], rb[32];
+            tmem_ld32(taddr + hb + c, ra);
+            tmem_ld32(taddr + hb + half + c, rb);
+            if (!row_ok) continue;
+            float va[32], vb[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const float2 cs = rope[c + i];
+                const float a = f32(ra[i]) * s, b = f32(rb[i]) * s;
+                va[i] = a * cs.x - b * cs.y;
+                vb[i] = b * cs.x + a * cs.y;
+            }
+            if (region == 0) {
+                bf16* op = ep.out + (size_t)row * ep.ld_out + n0 + hb + c;
+                store_bf16x32(op, va);
+                store_bf16x32(op + half, vb);
+            } else {
+                const int n = n0 + hb - ep.q_cols;
+                const int g = n / dh;
+                bf16* kp = ep.kcache + ((size_t)g * ep.max_ctx + pos) * dh + c;
+                store_bf16x32(kp, va);
+                store_bf16x32(kp + half, vb);
+            }
+        }
+    }
+}
+
+template <int BN>
+VLA_DEV void epi_swiglu(uint32_t taddr, int row, int n0, const EpiParams& ep) {
+    constexpr int HALF = BN / 2;
+    const bool row_ok = row < ep.M;
+    const float s = row_ok ? ep.rinv[row] : 0.f;
+    const int f0 = (n0 / BN) * HALF;
+#pragma unroll 1
+    for (int c = 0; c < HALF; c += 32) {
+        uint32_t rg[32], ru[32];
+        tmem_ld32(taddr + c, rg);
+        tmem_ld32(taddr + HALF + c, ru);
+        if (!row_ok) continue;
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            const float g = f32(rg[i]) * s;
+            const float u = f32(ru[i]) * s;
+            v[i] = g / (1.0f + __expf(-g)) * u;
+        }
+        store_bf16x32(ep.out + (size_t)row * ep.ld_out + f0 + c, v);
+    }
+}
+
+// Bounded wait that also gives up when another role has aborted.
+VLA_DEV bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity)) {
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kWaitBudgetCycles) return false;
+    }
+    return true;
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
+                      int N, int K, EpiParams ep) {
+    using C = GemmCfg<BN>;
+    constexpr int STAGES = C::STAGES;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ volatile int s_abort;
+
+    const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
+    uint8_t* smem = smem_raw + pad;
+    uint8_t* sA = smem;
+    uint8_t* sB = smem + STAGES * C::A_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + STAGES;
+    uint64_t* tfull = bars + 2 * STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* mma_done = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int num_m = (M + kBM - 1) / kBM;
+    const int num_n = (N + BN - 1) / BN;
+    const int num_tiles = num_m * num_n;
+    const int num_kb = (K + kBK - 1) / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&tfull[a], 1);
+            mbar_init(&tempty[a], 128);
+        }
+        mbar_init(mma_done, 1);
+        s_abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer ----------------
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued = 0, issued_phase = 0;  // per-stage bit masks of loads in flight
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+                const int m0 = (tile % num_m) * kBM;
+                const int n0 = (tile / num_m) * BN;
+                for (int kb = 0; kb < num_kb; ++kb) {
+                    if (!wait_or_abort(&empty[stage], phase ^ 1u, &s_abort)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+                    tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
+                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * kBK, n0);
+                    issued |= 1u << stage;
+                    issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                s_abort = 1;
+                set_status(ep.status, kDevTimeout);
+                // let every copy already issued land before the CTA can exit
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued & (1u << s)) mbar_wait(&full[s], (issued_phase >> s) & 1u);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            int it = 0;
+            for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++it) {
+                const int acc = it & 1;
+                const uint32_t acc_phase = (it >> 1) & 1;
+                if (!wait_or_abort(&tempty[acc], acc_phase ^ 1u, &s_abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + acc * BN;
+                for (int kb = 0; kb < num_kb; ++kb) {
+                    if (!wait_or_abort(&full[stage], phase, &s_abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t a_desc = sw128_kmajor_desc(smem_u32(sA + stage * C::A_BYTES));
+                    const uint64_t b_desc = sw128_kmajor_desc(smem_u32(sB + stage * C::B_BYTES));
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        // advance 16 bf16 (32 B) along K inside the 128-byte swizzle row
+                        umma_bf16_ss(d_tmem, a_desc + 2 * k, b_desc + 2 * k, C::IDESC, (kb | k) != 0);
+                    }
+                    umma_commit(&empty[stage]);
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (ok) umma_commit(&tfull[acc]);
+            }
+            if (!ok) {
+                s_abort = 1;
+                set_status(ep.status, kDevTimeout);
+            }
+            // all MMAs issued by this thread retire before TMEM can be released
+            umma_commit(mma_done);
+            mbar_wait(mma_done, 0);
+        }
+    } else {
+        // ---------------- epilogue (warps 2..5) ----------------
+        const int quarter = warp & 3;  // TMEM lanes [32*quarter, 32*quarter + 32)
+        int it = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
+            const int acc = it & 1;
+            const uint32_t acc_phase = (it >> 1) & 1;
+            const bool ok = wait_or_abort(&tfull[acc], acc_phase, &s_abort);
+            __syncwarp();
+            if (!__all_sync(0xFFFFFFFFu, ok)) {
+                s_abort = 1;
+                set_status(ep.status, kDevTimeout);
+                break;
+            }
+            tc_fence_after();
+            const int m0 = (tile % num_m) * kBM;
+            const int n0 = (tile / num_m) * BN;
+            const int row = m0 + quarter * 32 + lane;
+            const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+            if constexpr (EPI == kEpiQKV) {
+                epi_qkv<BN>(taddr, row, n0, ep);
+            } else if constexpr (EPI == kEpiSwiGLU) {
+                epi_swiglu<BN>(taddr, row, n0, ep);
+            } else {
+                epi_plain_resid<BN>(taddr, row, n0, ep);
+            }
+            tc_fence_before();
+            mbar_arrive(&tempty[acc]);
+        }
+    }
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, C::TMEM_COLS);
+    }
+}
+
+template <int BN, int EPI>
+cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K, const EpiParams& ep,
+                       int num_sms, cudaStream_t stream) {
+    using C = GemmCfg<BN>;
+    static bool attr_set = false;
+    auto kern = gemm_bf16_tcgen05<BN, EPI>;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
+    const int grid = tiles < num_sms ? tiles : num_sms;
+    kern<<<grid, kThreads, C::SMEM_BYTES, stream>>>(A, B, M, N, K, ep);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
+                        const EpiParams& ep, int num_sms, cudaStream_t stream) {
+    if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
+    if (bn == 256) {
+        switch (mode) {
+            case kEpiPlain:
+            case kEpiResid: return launch_one<256, kEpiResid>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream);
+        }
+    } else if (bn == 128) {
+        switch (mode) {
+            case kEpiPlain:
+            case kEpiResid: return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiQKV: return launch_one<128, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiSwiGLU: return launch_one<128, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace vla

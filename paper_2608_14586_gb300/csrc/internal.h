@@ -1,0 +1,129 @@
+// Internal launch interface between the C-ABI runtime and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace vla {
+
+using bf16 = __nv_bfloat16;
+
+// ---------------------------------------------------------------------------------------
+// tcgen05 GEMM: C[M,N] = A[M,K] * B[N,K]^T with a fused epilogue
+// ---------------------------------------------------------------------------------------
+enum EpiMode : int {
+    kEpiPlain = 0,   // out = bf16(acc)
+    kEpiResid = 1,   // out = bf16(resid + acc)                       (O / down projections)
+    kEpiQKV = 2,     // acc * rinv -> RoPE(q, k); q -> out, k/v -> KV cache (QKV projection)
+    kEpiSwiGLU = 3,  // gate/up tiles interleaved by 128 columns: out = silu(g*rinv) * (u*rinv)
+};
+
+struct EpiParams {
+    int M, N;
+    bf16* out;
+    int ld_out;
+    const bf16* resid;
+    int ld_resid;
+    const float* rinv;  // per-row 1/rms
+    // QKV epilogue
+    bf16* kcache;        // layer base, [n_kv_heads][max_ctx][head_dim]
+    bf16* vcache;
+    const float2* rope;  // [max_ctx][head_dim/2] (cos, sin)
+    int pos0, max_ctx, head_dim, q_cols, kv_cols;
+    unsigned* status;
+};
+
+// Tensor-map helper (driver entry point fetched through the runtime). rows x cols bf16,
+// row stride in elements; box = box_rows x 64 columns, 128-byte swizzle, zero fill.
+bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride,
+                    uint32_t box_rows);
+
+// Launch: BN in {128, 256}. Returns a cudaError_t of the launch.
+cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
+                        const EpiParams& ep, int num_sms, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------------------
+// Prefill attention (causal GQA, flash-style online softmax)
+// ---------------------------------------------------------------------------------------
+struct AttnPrefillParams {
+    const bf16* q;  // [M, H*dh]
+    int ld_q;
+    const bf16* kc;  // layer base [Hkv][max_ctx][dh]
+    const bf16* vc;
+    bf16* out;  // [M, H*dh]
+    int ld_out;
+    int M, H, Hkv, head_dim, max_ctx, pos0;
+    float scale_log2;  // log2(e) / sqrt(dh)
+};
+cudaError_t launch_attn_prefill(const AttnPrefillParams& p, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------------------
+// Elementwise / setup kernels
+// ---------------------------------------------------------------------------------------
+// rinv[i] = 1 / sqrt(mean_d x[i,d]^2 + eps)
+cudaError_t launch_rowstat(const bf16* x, int M, int D, int ld, float eps, float* rinv, cudaStream_t stream);
+
+// cos/sin table [max_ctx][dh/2] from float64 angles pos * base^(-2j/dh)
+cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream);
+
+// Repacking of one layer's weights into the library's layouts (gains folded in).
+struct RepackSrc {
+    const bf16 *w_q, *w_k, *w_v, *w_o, *w_gate, *w_up, *w_down, *g_attn, *g_mlp;
+};
+struct RepackDst {
+    bf16* w_qkv;  // [H*dh + 2*Hkv*dh, D], rows of q | k | v, each column scaled by g_attn
+    bf16* w_o;    // [D, H*dh]
+    bf16* w_gu;   // [2*F_pad, D], 256-row groups = 128 gate rows then 128 up rows, scaled by g_mlp
+    bf16* w_d;    // [D, F_pad], columns >= F zero
+};
+cudaError_t launch_repack(const RepackSrc& s, const RepackDst& d, int D, int H, int Hkv, int dh, int F, int F_pad,
+                          cudaStream_t stream);
+
+cudaError_t launch_set_lengths(int* d_len, int count, int value, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------------------
+// Decode (one token): weight-streaming GEMVs and split-KV attention
+// ---------------------------------------------------------------------------------------
+struct DecodeLayer {
+    const bf16 *w_qkv, *w_o, *w_gu, *w_d;
+    bf16* kcache;  // layer base [Hkv][max_ctx][dh]
+    bf16* vcache;
+    const int* d_len;  // this layer's device length (position of the new token)
+};
+struct DecodeDims {
+    int D, H, Hkv, dh, F_pad, max_ctx;
+    float eps;
+};
+struct DecodeWork {
+    float* q;          // [H*dh] fp32 (post-RoPE query)
+    float* part_o;     // [splits][H][dh]
+    float* part_ml;    // [splits][H][2]
+    bf16* attn;        // [H*dh]
+    bf16* x_mid;       // [D]
+    bf16* m;           // [F_pad]
+    const float2* rope;
+    unsigned* status;
+    int splits;
+};
+// Optional per-launch hook (measurement): called with (ctx, stage, begin) around each kernel.
+struct StageHook {
+    void (*fn)(void* ctx, int stage, bool begin);
+    void* ctx;
+    void operator()(int stage, bool begin) const {
+        if (fn) fn(ctx, stage, begin);
+    }
+};
+
+// Stage ids of the decode kernels (match VLA_STAGE_DEC_* in vla_prefix.h)
+enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecCombine = 9, kStageDecO = 10, kStageDecGateUp = 11,
+             kStageDecDown = 12 };
+
+cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
+                                bf16* x_out, int num_sms, bool pdl, cudaStream_t stream, const StageHook& hook);
+
+// d_len[i] += 1 for i < count (after all layers of a decode step have read their position)
+cudaError_t launch_advance_lengths(int* d_len, int count, bool pdl, cudaStream_t stream);
+
+}  // namespace vla
