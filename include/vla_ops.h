@@ -33,6 +33,33 @@ vla_status vla_op_attention_prefill(const void* q, const void* k_plane, const vo
                                     int n_heads, int n_kv_heads, int head_dim, int max_ctx, int pos0, void* out,
                                     vla_stream stream);
 
+/* Decode attention that allocates nothing. The paper has no counterpart: this entry point
+ * serves callers that may not allocate device memory while they run, such as a vehicle's
+ * real-time control loop that reserves all memory at start-up against a fixed budget (an
+ * allocation there can block for an unbounded time or fail), or a host framework whose own
+ * allocator owns the device memory.
+ *
+ * Computes, for one new token at position ctx-1, causal grouped-query attention over cache
+ * positions [0, ctx): out[h] = sum_j softmax_j(q_h . k_gj / sqrt(head_dim)) v_gj with
+ * g = h / (n_heads / n_kv_heads) — the same result vla_op_attention_prefill gives for
+ * n_tokens = 1 and pos0 = ctx - 1.
+ *   q        device bf16 [n_heads * head_dim] (post-rotary query)
+ *   k_plane, v_plane  device bf16 [n_kv_heads][max_ctx][head_dim], 16-byte aligned
+ *   out      device bf16 [n_heads * head_dim]
+ * head_dim in {64, 128}; n_heads / n_kv_heads in {1, 2, 4, 8}; 1 <= ctx <= max_ctx.
+ *
+ * Memory: the per-split partial results go to one 2 MiB array compiled into the library
+ * (present on every GPU that loads the library until the process exits); no call allocates
+ * or frees memory. Limit: n_heads * (head_dim + 2) <= 524288 floats (one split must fit),
+ * else VLA_ERR_SHAPE; the split count shrinks to fit the array. All calls share the array:
+ * calls whose GPU work overlaps (e.g. on different streams) race on it and must be ordered
+ * by the caller. The first call on a device resolves the array's device address (a
+ * cudaGetSymbolAddress with that device current) and reads its SM count; make that first
+ * call before any stream capture. Errors: INVALID_ARG, UNSUPPORTED, SHAPE, CUDA. */
+vla_status vla_op_attention_decode_noalloc(const void* q, const void* k_plane, const void* v_plane, int ctx,
+                                           int n_heads, int n_kv_heads, int head_dim, int max_ctx, void* out,
+                                           vla_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,7 +20,7 @@ __all__ = [
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_set_length", "vla_prefix_prefill",
     "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
-    "vla_prefix_stage_times", "STATUS", "STAGES",
+    "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "STATUS", "STAGES",
 ]
 
 # stage ids of vla_prefix_stage_times (VLA_STAGE_* in vla_prefix.h)
@@ -89,6 +89,7 @@ def load():
         "vla_op_gemm_bf16": ([V, V, I, I, I, V, V], I),
         "vla_op_attention_prefill": ([V, V, V, I, I, I, I, I, I, V, V], I),
         "vla_prefix_set_timing": ([P, I], I),
+        "vla_op_attention_decode_noalloc": ([V, V, V, I, I, I, I, I, V, V], I),
         "vla_prefix_stage_times": ([P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int), I], I),
     }
     for name, (args, res) in sig.items():
@@ -236,3 +237,11 @@ def vla_prefix_stage_times(p) -> dict:
     cnt = (ctypes.c_int * n)()
     _check(load().vla_prefix_stage_times(p, ms, cnt, n), "vla_prefix_stage_times")
     return {STAGES[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}
+
+
+def vla_op_attention_decode_noalloc(q, k_plane, v_plane, ctx: int, n_heads: int, n_kv_heads: int, head_dim: int,
+                                    max_ctx: int, out, stream=None):
+    """Decode attention whose scratch is a fixed array inside the library (no allocation)."""
+    _check(load().vla_op_attention_decode_noalloc(_ptr(q), _ptr(k_plane), _ptr(v_plane), ctx, n_heads, n_kv_heads,
+                                                  head_dim, max_ctx, _ptr(out), _stream(stream)),
+           "vla_op_attention_decode_noalloc")
