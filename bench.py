@@ -196,6 +196,21 @@ def to_dev(bits, torch):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
 
 
+def _traffic(kernel_key: str):
+    """DRAM bytes per launch of a kernel from the committed ncu summary, if it was taken on
+    the current source of that kernel (else None)."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            d = json.load(f)[kernel_key]
+        src = open(os.path.join(ROOT, d["source"]), "rb").read()
+        if hashlib.sha256(src).hexdigest()[:16] != d["source_sha256_16"]:
+            return None
+        return d["dram_bytes_per_launch"]
+    except Exception:
+        return None
+
+
 def run_ours(args, dist: Dist):
     import torch
 
@@ -208,14 +223,14 @@ def run_ours(args, dist: Dist):
     wl = synth.WORKLOADS[WORKLOAD]
     dwl = synth.WORKLOADS[DECODE_WORKLOAD]
     s = wl.shape
-    L = wl.prefix_layers
+    L = args.blocks or wl.prefix_layers
     M = wl.n_tokens
     D = s.hidden
     dec_steps = dwl.decode_steps
     max_ctx = max(M, dwl.prefill_ctx + dec_steps + 8)
     seed = wl.seed
 
-    # ---- model: the 16 prefix blocks (seeded synthetic weights), library-owned copies
+    # ---- model: the prefix blocks (seeded synthetic weights), library-owned copies
     layers = []
     for l in range(L):
         layers.append({k: to_dev(v, torch) for k, v in synth.layer_weights(s, seed, l).items()})
@@ -250,16 +265,17 @@ def run_ours(args, dist: Dist):
     for i in range(args.warmup):
         step(i, x)
     torch.cuda.synchronize()
-    vla.vla_prefix_stage_times(p)  # discard
 
     gpu_id = os.environ.get("CUDA_VISIBLE_DEVICES", str(dist.local)).split(",")[0] \
         if dist.world == 1 else str(dist.local)
     clocks = ClockSampler(gpu_id)
     clocks.start()
+    # ---- timed region: events bracket only the dominant kernel (gate/up GEMM)
     dist.barrier()
     torch.cuda.synchronize()
     launches[0] = 0
-    vla.vla_prefix_set_timing(p, True)
+    vla.vla_prefix_stage_times(p)
+    vla.vla_prefix_set_timing(p, ["gemm_gateup"])
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(main)
     for i in range(args.steps):
@@ -267,96 +283,120 @@ def run_ours(args, dist: Dist):
     main.wait_event(done[(args.steps - 1) & 1])
     t_end.record(main)
     torch.cuda.synchronize()
-    vla.vla_prefix_set_timing(p, False)
+    vla.vla_prefix_set_timing(p, ())
     dist.barrier()
     ms = t_start.elapsed_time(t_end) / args.steps
     ms = dist.max(ms, "cuda")
-    stages = vla.vla_prefix_stage_times(p)
+    gu_ms, gu_n = vla.vla_prefix_stage_times(p)["gemm_gateup"]
     prefill_launches = launches[0]
     assert vla.vla_last_async_error(p) == 0
 
+    # ---- diagnostic pass (not the timed region): every stage's average launch time
+    vla.vla_prefix_set_timing(p, "all")
+    for i in range(max(3, args.steps // 4)):
+        step(i, x)
+    torch.cuda.synchronize()
+    vla.vla_prefix_set_timing(p, ())
+    stages = vla.vla_prefix_stage_times(p)
+
     # roofline of the dominant kernel: gate/up projection + SwiGLU (51% of the GEMM flops)
-    gu_ms, gu_n = stages["gemm_gateup"]
     gu_flops = 2.0 * M * (2 * s.ffn) * D
     gu_tflops = gu_flops / (gu_ms / gu_n * 1e-3) / 1e12 if gu_n else 0.0
     block_flops = 2.0 * M * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
                              D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * M * M * s.head_dim * s.n_heads
     step_tflops = block_flops * L / (ms * 1e-3) / 1e12
 
-    # ---- end to end through the C ABI with host buffers (H2D of the frame, D2H of h^(16))
-    host_in = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).pin_memory()
-    x_dev = torch.empty_like(x)
+    # ---- end to end through the C ABI with host buffers (H2D of the frame, D2H of h^(k))
+    e2e = None
+    if not args.no_e2e:
+        host_in = torch.from_numpy(xb.view(np.int16)).view(torch.bfloat16).pin_memory()
+        x_dev = torch.empty_like(x)
 
-    def e2e_step(i):
-        b = i & 1
-        main.wait_event(done[b])
-        x_dev.copy_(host_in, non_blocking=True)
-        vla.vla_kv_reset(kv, main)
-        vla.vla_prefix_prefill(p, x_dev, M, 0, L, kv, outs[b], main)
-        ready[b].record(main)
-        vla.vla_boundary_to_host(outs[b], M, D, pinned[b], side, ready[b], done[b])
+        def e2e_step(i):
+            b = i & 1
+            main.wait_event(done[b])
+            x_dev.copy_(host_in, non_blocking=True)
+            vla.vla_kv_reset(kv, main)
+            vla.vla_prefix_prefill(p, x_dev, M, 0, L, kv, outs[b], main)
+            ready[b].record(main)
+            vla.vla_boundary_to_host(outs[b], M, D, pinned[b], side, ready[b], done[b])
 
-    for i in range(args.warmup):
-        e2e_step(i)
-    torch.cuda.synchronize()
-    dist.barrier()
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        e2e_step(i)
-    done[(args.steps - 1) & 1].synchronize()
-    torch.cuda.synchronize()
-    e2e_ms = (time.perf_counter() - t0) * 1e3 / args.steps
-    e2e_ms = dist.max(e2e_ms, "cuda")
-    # the boundary that reached the host equals the device result
-    assert torch.equal(pinned[(args.steps - 1) & 1].view(torch.int16).cpu(),
-                       outs[(args.steps - 1) & 1].view(torch.int16).cpu())
+        for i in range(args.warmup):
+            e2e_step(i)
+        torch.cuda.synchronize()
+        dist.barrier()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            e2e_step(i)
+        done[(args.steps - 1) & 1].synchronize()
+        torch.cuda.synchronize()
+        e2e_ms = (time.perf_counter() - t0) * 1e3 / args.steps
+        e2e_ms = dist.max(e2e_ms, "cuda")
+        # the boundary that reached the host equals the device result
+        assert torch.equal(pinned[(args.steps - 1) & 1].view(torch.int16).cpu(),
+                           outs[(args.steps - 1) & 1].view(torch.int16).cpu())
+        e2e = {"value": M * dist.world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": M * D * 2, "d2h_bytes_per_step": M * D * 2}
 
     # ---- decode: 64 single-token steps against a 2304-position random context
-    ctx0 = dwl.prefill_ctx
-    for l in range(L):
-        kb, vb = synth.random_kv(ctx0, s, dwl.seed, l)
-        kp, vp = vla.vla_kv_data(kv, l)
-        for ptr, bits in ((kp, kb), (vp, vb)):
-            src = to_dev(bits, torch)  # [Hkv, ctx0, dh] -> rows of the [Hkv, max_ctx, dh] plane
-            for g in range(s.n_kv_heads):
-                dst = _dev_view(ptr + g * max_ctx * s.head_dim * 2, ctx0 * s.head_dim, torch)
-                dst.copy_(src[g].reshape(-1))
-    torch.cuda.synchronize()
-    xd = to_dev(np.stack([synth.decode_hidden(t, D, dwl.seed)[0] for t in range(dec_steps)]), torch)
-    yd = torch.empty((1, D), dtype=torch.bfloat16, device="cuda")
+    decode = None
+    if not args.no_decode:
+        ctx0 = dwl.prefill_ctx
+        for l in range(L):
+            kb, vb = synth.random_kv(ctx0, s, dwl.seed, l)
+            kp, vp = vla.vla_kv_data(kv, l)
+            for ptr, bits in ((kp, kb), (vp, vb)):
+                src = to_dev(bits, torch)  # [Hkv, ctx0, dh] -> rows of the [Hkv, max_ctx, dh] plane
+                for g in range(s.n_kv_heads):
+                    dst = _dev_view(ptr + g * max_ctx * s.head_dim * 2, ctx0 * s.head_dim, torch)
+                    dst.copy_(src[g].reshape(-1))
+        torch.cuda.synchronize()
+        xd = to_dev(np.stack([synth.decode_hidden(t, D, dwl.seed)[0] for t in range(dec_steps)]), torch)
+        yd = torch.empty((1, D), dtype=torch.bfloat16, device="cuda")
 
-    def decode_run():
-        vla.vla_kv_set_length(kv, ctx0, main)
-        n = 1
-        for t in range(dec_steps):
-            vla.vla_prefix_decode(p, xd[t:t + 1], 0, L, kv, yd, main)
-            n += vla.vla_last_launch_count(p)
-        return n
+        def decode_run():
+            vla.vla_kv_set_length(kv, ctx0, main)
+            n = 1
+            for t in range(dec_steps):
+                vla.vla_prefix_decode(p, xd[t:t + 1], 0, L, kv, yd, main)
+                n += vla.vla_last_launch_count(p)
+            return n
 
-    for _ in range(max(1, args.warmup // 2)):
+        for _ in range(max(1, args.warmup // 2)):
+            decode_run()
+        torch.cuda.synchronize()
+        dist.barrier()
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        d0.record(main)
+        reps = max(1, args.steps // 8)
+        dec_launches = 0
+        for _ in range(reps):
+            dec_launches += decode_run()
+        d1.record(main)
+        torch.cuda.synchronize()
+        dist.barrier()
+        dec_us = d0.elapsed_time(d1) * 1e3 / (reps * dec_steps)
+        dec_us = dist.max(dec_us, "cuda")
+        assert vla.vla_last_async_error(p) == 0
+        vla.vla_prefix_set_timing(p, "all")
         decode_run()
-    torch.cuda.synchronize()
-    dist.barrier()
-    vla.vla_prefix_stage_times(p)
-    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    d0.record(main)
-    reps = max(1, args.steps // 8)
-    dec_launches = 0
-    for _ in range(reps):
-        dec_launches += decode_run()
-    d1.record(main)
-    torch.cuda.synchronize()
+        torch.cuda.synchronize()
+        vla.vla_prefix_set_timing(p, ())
+        dstages = vla.vla_prefix_stage_times(p)
+        weight_bytes = L * 2 * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                                D * s.n_heads * s.head_dim + 3 * s.ffn * D)
+        avg_ctx = ctx0 + (dec_steps + 1) / 2
+        kv_bytes = L * 2 * s.n_kv_heads * s.head_dim * 2 * avg_ctx
+        dec_bytes = weight_bytes + kv_bytes
+        dec_gbs = dec_bytes / (dec_us * 1e-6) / 1e9
+        decode = {"workload": DECODE_WORKLOAD, "blocks": L, "us_per_step": dec_us, "bytes_per_step": dec_bytes,
+                  "hbm_gbs": dec_gbs,
+                  "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm_peak, "unit": "GB/s",
+                               "frac": dec_gbs / hbm_peak, "peak_source": f"{peak_src} copy bandwidth",
+                               "traffic": None},
+                  "gpu_launches_per_step": dec_launches / (reps * dec_steps),
+                  "stages_us_per_launch": {k: round(v[0] / v[1] * 1e3, 2) for k, v in dstages.items() if v[1]}}
     clock_info = clocks.stop()
-    dist.barrier()
-    dec_us = d0.elapsed_time(d1) * 1e3 / (reps * dec_steps)
-    dec_us = dist.max(dec_us, "cuda")
-    assert vla.vla_last_async_error(p) == 0
-    weight_bytes = L * 2 * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
-                            D * s.n_heads * s.head_dim + 3 * s.ffn * D)
-    avg_ctx = ctx0 + (dec_steps + 1) / 2
-    kv_bytes = L * 2 * s.n_kv_heads * s.head_dim * 2 * avg_ctx
-    dec_bytes = weight_bytes + kv_bytes
-    dec_gbs = dec_bytes / (dec_us * 1e-6) / 1e9
 
     # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame
     cpu = None
@@ -372,27 +412,22 @@ def run_ours(args, dist: Dist):
             "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": dist.world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "blocks": L, "tokens": M, "hidden": D,
+            "config": {"workload": WORKLOAD if L == wl.prefix_layers else f"{WORKLOAD} ({L} blocks)",
+                       "blocks": L, "tokens": M, "hidden": D,
                        "heads": f"{s.n_heads}q/{s.n_kv_heads}kv x {s.head_dim}", "ffn": s.ffn,
                        "boundary_bytes": M * D * 2, "l2": "weights 5.67 GB streamed per step > 129 MB L2",
                        "parallelism": f"replicas x{dist.world}"},
             "roofline": {"kernel": "gemm_gateup (tcgen05, SwiGLU epilogue)", "bound": "tensor",
                          "achieved": gu_tflops, "peak": bf16_sust, "unit": "TFLOP/s", "frac": gu_tflops / bf16_sust,
-                         "peak_source": f"{peak_src} bf16 sustained", "traffic": None,
+                         "peak_source": f"{peak_src} bf16 sustained", "traffic": _traffic("gemm_gateup"),
                          "flops_per_launch": gu_flops, "avg_launch_ms": gu_ms / max(gu_n, 1)},
             "step_tflops": step_tflops, "step_frac_of_peak": step_tflops / bf16_sust,
             "cpu_baseline": cpu,
-            "e2e": {"value": M * dist.world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
-                    "h2d_bytes_per_step": M * D * 2, "d2h_bytes_per_step": M * D * 2},
+            "e2e": e2e,
             "gpu_launches": prefill_launches,
             "clocks": clock_info,
             "stages_ms_per_launch": {k: round(v[0] / v[1], 4) for k, v in stages.items() if v[1]},
-            "decode": {"workload": DECODE_WORKLOAD, "us_per_step": dec_us, "bytes_per_step": dec_bytes,
-                       "hbm_gbs": dec_gbs, "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm_peak,
-                                                        "unit": "GB/s", "frac": dec_gbs / hbm_peak,
-                                                        "peak_source": f"{peak_src} copy bandwidth",
-                                                        "traffic": None},
-                       "gpu_launches_per_step": dec_launches / (reps * dec_steps)},
+            "decode": decode,
         }
         print(json.dumps(line), flush=True)
     vla.vla_kv_destroy(kv)
@@ -417,6 +452,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--blocks", type=int, default=0, help="prefix depth (default: the workload's 16)")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

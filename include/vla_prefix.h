@@ -152,8 +152,9 @@ const char* vla_status_str(vla_status s);
 /* Number of kernels the last prefill / decode call of `p` enqueued (for launch accounting). */
 int vla_last_launch_count(const vla_prefix* p);
 
-/* Measurement support (not part of the method): when enabled, prefill and decode record a
- * CUDA event pair around every kernel they enqueue, on the call's stream.
+/* Measurement support (not part of the method): prefill and decode record a CUDA event pair
+ * on the call's stream around every kernel of a stage whose bit (1 << stage id) is set in
+ * the mask given to vla_prefix_set_timing (0 turns timing off).
  * vla_prefix_stage_times synchronises those events and returns, per stage id below, the
  * summed kernel time in milliseconds and the number of launches since the last read, then
  * clears them. Arrays have n_stages entries (VLA_STAGE_COUNT covers all). */
@@ -173,7 +174,7 @@ enum {
     VLA_STAGE_DEC_DOWN = 12,    /* decode: down projection + residual            */
     VLA_STAGE_COUNT = 13
 };
-vla_status vla_prefix_set_timing(vla_prefix* p, int enable);
+vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask);
 vla_status vla_prefix_stage_times(vla_prefix* p, float* ms_per_stage, int* launches_per_stage, int n_stages);
 
 #ifdef __cplusplus

@@ -88,7 +88,7 @@ def load():
         "vla_last_launch_count": ([P], I),
         "vla_op_gemm_bf16": ([V, V, I, I, I, V, V], I),
         "vla_op_attention_prefill": ([V, V, V, I, I, I, I, I, I, V, V], I),
-        "vla_prefix_set_timing": ([P, I], I),
+        "vla_prefix_set_timing": ([P, ctypes.c_uint], I),
         "vla_op_attention_decode_noalloc": ([V, V, V, I, I, I, I, I, V, V], I),
         "vla_prefix_stage_times": ([P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int), I], I),
     }
@@ -226,8 +226,14 @@ def vla_op_attention_prefill(q, k_plane, v_plane, n_tokens: int, n_heads: int, n
            "vla_op_attention_prefill")
 
 
-def vla_prefix_set_timing(p, enable: bool):
-    _check(load().vla_prefix_set_timing(p, 1 if enable else 0), "vla_prefix_set_timing")
+def vla_prefix_set_timing(p, stages=()):
+    """Time the kernels of the named stages (an iterable of STAGES names, or "all"); () = off."""
+    if stages == "all":
+        stages = STAGES
+    mask = 0
+    for name in stages:
+        mask |= 1 << STAGES.index(name)
+    _check(load().vla_prefix_set_timing(p, mask), "vla_prefix_set_timing")
 
 
 def vla_prefix_stage_times(p) -> dict:

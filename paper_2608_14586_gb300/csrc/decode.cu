@@ -9,8 +9,8 @@
 //     SwiGLU, consecutive rows for the residual projections;
 //   * the input vector is staged in shared memory; RMSNorm's 1/rms is computed per CTA
 //     (the gains are folded into the weights);
-//   * launched with programmatic dependent launch: each kernel prefetches its first weight
-//     rows into L2 before griddepcontrol.wait, overlapping the previous kernel's tail.
+//   * each kernel prefetches its first weight rows into L2 before reading its input vector,
+//     so the weight stream starts while the input is still being staged.
 // Attention is split over the context (fixed split count -> deterministic): each CTA owns
 // one KV head (all query heads of its GQA group) and a contiguous key range, 8 lanes per key
 // row, online softmax in fp32; a combine kernel merges the partial (max, sum, output).
@@ -129,9 +129,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pb + l * 128));
         }
     }
-    pdl_trigger();
-    pdl_wait();
-
     const uint4* xg = reinterpret_cast<const uint4*>(p.xv);
     for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) xs[i] = xg[i];
     __syncthreads();
@@ -213,8 +210,6 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_partial_kernel(AttnD
     const int kvh = blockIdx.x, split = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane >> 3, l8 = lane & 7;
-    pdl_trigger();
-    pdl_wait();
     const int ctx = *p.d_len + 1;
     const int chunk = (ctx + p.splits - 1) / p.splits;
     const int kb = split * chunk;
@@ -339,8 +334,6 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_partial_kernel(AttnD
 // out[h*dh + d] = sum_s o_s e^(m_s - M) / sum_s l_s e^(m_s - M)   (fixed split order)
 __global__ void attn_decode_combine_kernel(const float* part_o, const float* part_ml, int H, int dh, int splits,
                                            bf16* out) {
-    pdl_trigger();
-    pdl_wait();
     const int h = blockIdx.x;
     for (int d = threadIdx.x; d < dh; d += blockDim.x) {
         float mx = -INFINITY;
@@ -358,30 +351,12 @@ __global__ void attn_decode_combine_kernel(const float* part_o, const float* par
 }
 
 __global__ void advance_lengths_kernel(int* d_len, int count) {
-    pdl_trigger();
-    pdl_wait();
     const int i = threadIdx.x;
     if (i < count) d_len[i] += 1;
 }
 
-template <typename... KArgs, typename... Args>
-cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, bool pdl, cudaStream_t s,
-                     Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, kern, args...);
-}
-
 template <int MODE>
-cudaError_t launch_gemv(const GemvParams& p, int num_sms, bool pdl, cudaStream_t s) {
+cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s) {
     const size_t smem = (size_t)p.K * 2;
     static bool attr_set = false;
     if (!attr_set) {
@@ -393,28 +368,30 @@ cudaError_t launch_gemv(const GemvParams& p, int num_sms, bool pdl, cudaStream_t
     int grid = 2 * num_sms;
     const int gmax = (warps_needed + 7) / 8;
     if (grid > gmax) grid = gmax;
-    return launch_k(gemv_kernel<MODE>, dim3(grid), dim3(kGemvThreads), smem, pdl, s, p);
+    gemv_kernel<MODE><<<grid, kGemvThreads, smem, s>>>(p);
+    return cudaGetLastError();
 }
 
 template <int DH, int G>
-cudaError_t launch_attn_dec(const AttnDecParams& p, bool pdl, cudaStream_t s) {
-    return launch_k(attn_decode_partial_kernel<DH, G>, dim3(p.Hkv, p.splits), dim3(kAttnThreads), 0, pdl, s, p);
+cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s) {
+    attn_decode_partial_kernel<DH, G><<<dim3(p.Hkv, p.splits), kAttnThreads, 0, s>>>(p);
+    return cudaGetLastError();
 }
 
-cudaError_t launch_attn_dec_any(int dh, int group, const AttnDecParams& p, bool pdl, cudaStream_t s) {
+cudaError_t launch_attn_dec_any(int dh, int group, const AttnDecParams& p, cudaStream_t s) {
     if (dh == 128) {
         switch (group) {
-            case 1: return launch_attn_dec<128, 1>(p, pdl, s);
-            case 2: return launch_attn_dec<128, 2>(p, pdl, s);
-            case 4: return launch_attn_dec<128, 4>(p, pdl, s);
-            case 8: return launch_attn_dec<128, 8>(p, pdl, s);
+            case 1: return launch_attn_dec<128, 1>(p, s);
+            case 2: return launch_attn_dec<128, 2>(p, s);
+            case 4: return launch_attn_dec<128, 4>(p, s);
+            case 8: return launch_attn_dec<128, 8>(p, s);
         }
     } else if (dh == 64) {
         switch (group) {
-            case 1: return launch_attn_dec<64, 1>(p, pdl, s);
-            case 2: return launch_attn_dec<64, 2>(p, pdl, s);
-            case 4: return launch_attn_dec<64, 4>(p, pdl, s);
-            case 8: return launch_attn_dec<64, 8>(p, pdl, s);
+            case 1: return launch_attn_dec<64, 1>(p, s);
+            case 2: return launch_attn_dec<64, 2>(p, s);
+            case 4: return launch_attn_dec<64, 4>(p, s);
+            case 8: return launch_attn_dec<64, 8>(p, s);
         }
     }
     return cudaErrorInvalidValue;
@@ -423,7 +400,7 @@ cudaError_t launch_attn_dec_any(int dh, int group, const AttnDecParams& p, bool 
 }  // namespace
 
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
-                                bf16* x_out, int num_sms, bool pdl, cudaStream_t stream, const StageHook& hook) {
+                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook) {
     cudaError_t e;
     const int qc = d.H * d.dh, kvc = d.Hkv * d.dh;
     // 1. RMSNorm + QKV + RoPE + KV append
@@ -443,7 +420,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     g.max_ctx = d.max_ctx;
     g.eps = d.eps;
     hook(kStageDecQKV, true);
-    e = launch_gemv<kGemvQKV>(g, num_sms, pdl, stream);
+    e = launch_gemv<kGemvQKV>(g, num_sms, stream);
     hook(kStageDecQKV, false);
     if (e != cudaSuccess) return e;
     // 2. split-KV attention + combine
@@ -460,12 +437,12 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     a.part_o = w.part_o;
     a.part_ml = w.part_ml;
     hook(kStageDecAttn, true);
-    e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, pdl, stream);
+    e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, stream);
     hook(kStageDecAttn, false);
     if (e != cudaSuccess) return e;
     hook(kStageDecCombine, true);
-    e = launch_k(attn_decode_combine_kernel, dim3(d.H), dim3(d.dh), 0, pdl, stream, (const float*)w.part_o,
-                 (const float*)w.part_ml, d.H, d.dh, w.splits, w.attn);
+    attn_decode_combine_kernel<<<d.H, d.dh, 0, stream>>>(w.part_o, w.part_ml, d.H, d.dh, w.splits, w.attn);
+    e = cudaGetLastError();
     hook(kStageDecCombine, false);
     if (e != cudaSuccess) return e;
     // 3. O projection + residual
@@ -477,7 +454,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     o.resid = x_in;
     o.out = w.x_mid;
     hook(kStageDecO, true);
-    e = launch_gemv<kGemvResid>(o, num_sms, pdl, stream);
+    e = launch_gemv<kGemvResid>(o, num_sms, stream);
     hook(kStageDecO, false);
     if (e != cudaSuccess) return e;
     // 4. RMSNorm + gate/up + SwiGLU
@@ -489,7 +466,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     gu.out = w.m;
     gu.eps = d.eps;
     hook(kStageDecGateUp, true);
-    e = launch_gemv<kGemvSwiGLU>(gu, num_sms, pdl, stream);
+    e = launch_gemv<kGemvSwiGLU>(gu, num_sms, stream);
     hook(kStageDecGateUp, false);
     if (e != cudaSuccess) return e;
     // 5. down projection + residual
@@ -501,14 +478,15 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     dn.resid = w.x_mid;
     dn.out = x_out;
     hook(kStageDecDown, true);
-    e = launch_gemv<kGemvResid>(dn, num_sms, pdl, stream);
+    e = launch_gemv<kGemvResid>(dn, num_sms, stream);
     hook(kStageDecDown, false);
     return e;
 }
 
-cudaError_t launch_advance_lengths(int* d_len, int count, bool pdl, cudaStream_t stream) {
+cudaError_t launch_advance_lengths(int* d_len, int count, cudaStream_t stream) {
     if (count <= 0) return cudaSuccess;
-    return launch_k(advance_lengths_kernel, dim3(1), dim3(((count + 31) / 32) * 32), 0, pdl, stream, d_len, count);
+    advance_lengths_kernel<<<1, ((count + 31) / 32) * 32, 0, stream>>>(d_len, count);
+    return cudaGetLastError();
 }
 
 }  // namespace vla

@@ -121,9 +121,9 @@ enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecCombine = 9, kStageDe
              kStageDecDown = 12 };
 
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
-                                bf16* x_out, int num_sms, bool pdl, cudaStream_t stream, const StageHook& hook);
+                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook);
 
 // d_len[i] += 1 for i < count (after all layers of a decode step have read their position)
-cudaError_t launch_advance_lengths(int* d_len, int count, bool pdl, cudaStream_t stream);
+cudaError_t launch_advance_lengths(int* d_len, int count, cudaStream_t stream);
 
 }  // namespace vla

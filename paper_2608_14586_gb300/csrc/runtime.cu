@@ -11,7 +11,7 @@
 //   GEMM  m * Wd^T     [kEpiResid]     x_out = x_mid + m Wd^T -> hidden_out
 // Block b reads hidden_in; later blocks work in place in hidden_out, so the range needs one
 // extra [M, D] buffer (x_mid). hidden_out after the last block is h^(layer_end) (Eq. 5).
-// Decode runs the same stages as GEMVs (decode.cu).
+// Decode runs the same stages as GEMVs (decode.cu), replayed as a CUDA graph per step.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -74,11 +74,12 @@ namespace {
 
 constexpr int kBN = 256;  // N tile of every prefill GEMM
 
-// Decode kernels are launched in plain stream order. (They are written so programmatic
-// dependent launch could overlap each kernel's weight prefetch with its predecessor, but a
-// decode step launched that way on the legacy default stream did not complete; until that
-// is understood the attribute stays off.)
-constexpr bool kDecodePDL = false;
+// A decode step is ~6 kernels per block (~97 for 16 blocks), each only a few to a few tens
+// of microseconds long, so host launch cost would dominate. The step is captured once per
+// (KV cache, layer range) as a CUDA graph that reads the token from a library-owned staging
+// vector and the position from the cache's device-side lengths; every later step is one
+// graph launch plus two 8 KB device copies in/out of the staging vectors.
+constexpr int kMaxDecodeGraphs = 8;
 
 struct LayerDev {
     bf16 *w_qkv, *w_o, *w_gu, *w_d;
@@ -105,7 +106,7 @@ struct vla_prefix {
     unsigned* d_status = nullptr;
     int last_launches = 0;
     // measurement: event pairs around each kernel while timing is enabled
-    bool timing = false;
+    unsigned timing = 0;  // bit s: time the kernels of stage s
     std::vector<cudaEvent_t> ev_pool;
     size_t ev_used = 0;
     struct Rec {
@@ -115,6 +116,15 @@ struct vla_prefix {
     std::vector<Rec> recs;
     cudaStream_t cur_stream = nullptr;
     cudaEvent_t pending = nullptr;
+    // decode graphs
+    bf16 *d_xin = nullptr, *d_xout = nullptr;  // [D] staging vectors of a decode step
+    cudaStream_t cap_stream = nullptr;
+    struct DecodeGraph {
+        const vla_kv* kv;
+        int lb, le;
+        cudaGraphExec_t exec;
+    };
+    std::vector<DecodeGraph> graphs;
 };
 
 struct vla_kv {
@@ -154,6 +164,10 @@ void free_prefix(vla_prefix* p) {
     cudaFree(p->d_m);
     cudaFree(p->d_status);
     for (cudaEvent_t e : p->ev_pool) cudaEventDestroy(e);
+    for (auto& g : p->graphs) cudaGraphExecDestroy(g.exec);
+    if (p->cap_stream) cudaStreamDestroy(p->cap_stream);
+    cudaFree(p->d_xin);
+    cudaFree(p->d_xout);
     delete p;
 }
 
@@ -168,7 +182,7 @@ cudaEvent_t pool_event(vla_prefix* p) {
 
 // Records the start / end event of one kernel of `stage` when timing is enabled.
 void stage_mark(vla_prefix* p, int stage, bool begin) {
-    if (!p->timing) return;
+    if (!(p->timing & (1u << stage))) return;
     if (begin) {
         p->pending = pool_event(p);
         if (p->pending) cudaEventRecord(p->pending, p->cur_stream);
@@ -272,7 +286,8 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
               dmalloc(&p->ws_rinv, (size_t)T) && dmalloc(&p->dq, (size_t)p->qc) &&
               dmalloc(&p->d_part_o, (size_t)p->dec_splits * H * dh) &&
               dmalloc(&p->d_part_ml, (size_t)p->dec_splits * H * 2) && dmalloc(&p->d_attn, (size_t)p->qc) &&
-              dmalloc(&p->d_xmid, (size_t)D) && dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1);
+              dmalloc(&p->d_xmid, (size_t)D) && dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1) &&
+              dmalloc(&p->d_xin, (size_t)D) && dmalloc(&p->d_xout, (size_t)D);
     if (!ok) {
         cudaGetLastError();
         free_prefix(p);
@@ -355,6 +370,15 @@ vla_status vla_kv_create(vla_prefix* p, int layer_begin, int layer_end, int max_
 vla_status vla_kv_destroy(vla_kv* kv) {
     if (!kv) return VLA_OK;
     cudaDeviceSynchronize();
+    auto& gs = kv->p->graphs;
+    for (size_t i = 0; i < gs.size();) {
+        if (gs[i].kv == kv) {
+            cudaGraphExecDestroy(gs[i].exec);
+            gs.erase(gs.begin() + i);
+        } else {
+            ++i;
+        }
+    }
     cudaFree(kv->data);
     cudaFree(kv->d_len);
     delete kv;
@@ -533,26 +557,59 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
                             p->cfg.rms_eps};
     vla::DecodeWork w = {p->dq, p->d_part_o, p->d_part_ml, p->d_attn, p->d_xmid, p->d_m, p->rope, p->d_status,
                          p->dec_splits};
+    const int nl = layer_end - layer_begin;
+    // enqueue the whole step on stream s, reading x_in and chaining through x_out
+    auto enqueue = [&](const bf16* x_in, bf16* x_out, cudaStream_t s, const vla::StageHook& hook) {
+        cudaError_t e = cudaSuccess;
+        for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
+            const LayerDev& ld = p->layers[l];
+            vla::DecodeLayer L = {ld.w_qkv, ld.w_o, ld.w_gu, ld.w_d, kv->k_plane(l), kv->v_plane(l),
+                                  kv->d_len + (l - kv->lb)};
+            e = vla::launch_decode_layer(L, dims, w, l == layer_begin ? x_in : x_out, x_out, p->num_sms, s, hook);
+        }
+        if (e == cudaSuccess) e = vla::launch_advance_lengths(kv->d_len + (layer_begin - kv->lb), nl, s);
+        return e;
+    };
     cudaError_t e = cudaSuccess;
-    int launches = 0;
     p->cur_stream = stream;
-    const vla::StageHook hook = {p->timing ? stage_hook_fn : nullptr, p};
-    for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
-        const LayerDev& ld = p->layers[l];
-        vla::DecodeLayer L = {ld.w_qkv, ld.w_o, ld.w_gu, ld.w_d, kv->k_plane(l), kv->v_plane(l),
-                              kv->d_len + (l - kv->lb)};
-        const bf16* x = (l == layer_begin) ? (const bf16*)hidden_in : (const bf16*)hidden_out;
-        e = vla::launch_decode_layer(L, dims, w, x, (bf16*)hidden_out, p->num_sms, kDecodePDL, stream, hook);
-        launches += 6;
+    if (p->timing) {
+        // measurement mode: direct launches with event pairs around the selected stages
+        const vla::StageHook hook = {stage_hook_fn, p};
+        e = enqueue((const bf16*)hidden_in, (bf16*)hidden_out, stream, hook);
+    } else {
+        cudaGraphExec_t exec = nullptr;
+        for (const auto& g : p->graphs)
+            if (g.kv == kv && g.lb == layer_begin && g.le == layer_end) exec = g.exec;
+        if (!exec) {
+            if (!p->cap_stream && cudaStreamCreateWithFlags(&p->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+                return VLA_ERR_CUDA;
+            cudaGraph_t graph = nullptr;
+            e = cudaStreamBeginCapture(p->cap_stream, cudaStreamCaptureModeRelaxed);
+            if (e == cudaSuccess) {
+                cudaError_t le = enqueue(p->d_xin, p->d_xout, p->cap_stream, vla::StageHook{nullptr, nullptr});
+                e = cudaStreamEndCapture(p->cap_stream, &graph);
+                if (le != cudaSuccess) e = le;
+            }
+            if (e == cudaSuccess) e = cudaGraphInstantiate(&exec, graph, 0);
+            if (graph) cudaGraphDestroy(graph);
+            if (e != cudaSuccess) {
+                cudaGetLastError();
+                return VLA_ERR_CUDA;
+            }
+            if ((int)p->graphs.size() >= kMaxDecodeGraphs) {
+                cudaGraphExecDestroy(p->graphs.front().exec);
+                p->graphs.erase(p->graphs.begin());
+            }
+            p->graphs.push_back({kv, layer_begin, layer_end, exec});
+        }
+        e = cudaMemcpyAsync(p->d_xin, hidden_in, (size_t)D * 2, cudaMemcpyDeviceToDevice, stream);
+        if (e == cudaSuccess) e = cudaGraphLaunch(exec, stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(hidden_out, p->d_xout, (size_t)D * 2, cudaMemcpyDeviceToDevice, stream);
     }
-    stage_mark(p, VLA_STAGE_KV_LEN, true);
-    if (e == cudaSuccess)
-        e = vla::launch_advance_lengths(kv->d_len + (layer_begin - kv->lb), layer_end - layer_begin, kDecodePDL,
-                                         stream);
-    stage_mark(p, VLA_STAGE_KV_LEN, false);
     if (e != cudaSuccess) return VLA_ERR_CUDA;
     for (int l = layer_begin; l < layer_end; ++l) kv->len[l - kv->lb] = p0 + 1;
-    p->last_launches = launches + 1;
+    p->last_launches = 6 * nl + 1;
     return VLA_OK;
 }
 
@@ -584,9 +641,9 @@ vla_status vla_last_async_error(vla_prefix* p) {
 
 int vla_last_launch_count(const vla_prefix* p) { return p ? p->last_launches : 0; }
 
-vla_status vla_prefix_set_timing(vla_prefix* p, int enable) {
+vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask) {
     if (!p) return VLA_ERR_INVALID_ARG;
-    p->timing = enable != 0;
+    p->timing = stage_mask;
     return VLA_OK;
 }
 
