@@ -40,12 +40,17 @@ struct EpiParams {
 bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride,
                     uint32_t box_rows);
 
+// 3-D bf16 map: [planes][rows][inner] with rows of `inner` elements and planes
+// `plane_stride` elements apart; box = 1 plane x box_rows x 64, 128-byte swizzle, zero fill.
+bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t planes,
+                       uint64_t plane_stride, uint32_t box_rows);
+
 // Launch: BN in {128, 256}. Returns a cudaError_t of the launch.
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
                         const EpiParams& ep, int num_sms, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------------------
-// Prefill attention (causal GQA, flash-style online softmax)
+// Prefill attention (causal GQA, flash-style online softmax, attention_tc.cu)
 // ---------------------------------------------------------------------------------------
 struct AttnPrefillParams {
     const bf16* q;  // [M, H*dh]
@@ -57,7 +62,8 @@ struct AttnPrefillParams {
     int M, H, Hkv, head_dim, max_ctx, pos0;
     float scale_log2;  // log2(e) / sqrt(dh)
 };
-cudaError_t launch_attn_prefill(const AttnPrefillParams& p, cudaStream_t stream);
+// tcgen05 kernel (S and O in tensor memory); `status` receives a timeout code
+cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------------------
 // Elementwise / setup kernels

@@ -61,6 +61,20 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
     return r == CUDA_SUCCESS;
 }
 
+bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t planes,
+                       uint64_t plane_stride, uint32_t box_rows) {
+    PFN_encodeTiled_t enc = get_encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {inner, rows, planes};
+    cuuint64_t strides[2] = {inner * 2, plane_stride * 2};
+    cuuint32_t box[3] = {64, box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 static int device_sm_count() {
     int dev = 0, n = 0;
     cudaGetDevice(&dev);
@@ -484,7 +498,7 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ap.pos0 = p0;
         ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)p->cfg.head_dim));
         stage_mark(p, VLA_STAGE_ATTN, true);
-        e = vla::launch_attn_prefill(ap, stream);
+        e = vla::launch_attn_prefill_tc(ap, p->d_status, stream);
         stage_mark(p, VLA_STAGE_ATTN, false);
         if (e != cudaSuccess) break;
         // output projection + residual
@@ -716,7 +730,7 @@ vla_status vla_op_attention_prefill(const void* q, const void* k_plane, const vo
     ap.max_ctx = max_ctx;
     ap.pos0 = pos0;
     ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
-    return cuda_status(vla::launch_attn_prefill(ap, (cudaStream_t)stream));
+    return cuda_status(vla::launch_attn_prefill_tc(ap, nullptr, (cudaStream_t)stream));
 }
 
 }  // extern "C"
