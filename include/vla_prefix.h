@@ -167,12 +167,11 @@ enum {
     VLA_STAGE_GEMM_DOWN = 5,    /* down projection + residual (prefill)         */
     VLA_STAGE_KV_LEN = 6,       /* KV length update                              */
     VLA_STAGE_DEC_QKV = 7,      /* decode: RMSNorm + QKV + RoPE + KV append      */
-    VLA_STAGE_DEC_ATTN = 8,     /* decode: split-KV attention partials           */
-    VLA_STAGE_DEC_COMBINE = 9,  /* decode: split combine                          */
-    VLA_STAGE_DEC_O = 10,       /* decode: output projection + residual          */
-    VLA_STAGE_DEC_GATEUP = 11,  /* decode: RMSNorm + gate/up + SwiGLU            */
-    VLA_STAGE_DEC_DOWN = 12,    /* decode: down projection + residual            */
-    VLA_STAGE_COUNT = 13
+    VLA_STAGE_DEC_ATTN = 8,     /* decode: split-KV attention + merge            */
+    VLA_STAGE_DEC_O = 9,        /* decode: output projection + residual          */
+    VLA_STAGE_DEC_GATEUP = 10,  /* decode: RMSNorm + gate/up + SwiGLU            */
+    VLA_STAGE_DEC_DOWN = 11,    /* decode: down projection + residual            */
+    VLA_STAGE_COUNT = 12
 };
 vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask);
 vla_status vla_prefix_stage_times(vla_prefix* p, float* ms_per_stage, int* launches_per_stage, int n_stages);

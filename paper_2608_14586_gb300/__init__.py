@@ -25,7 +25,7 @@ __all__ = [
 
 # stage ids of vla_prefix_stage_times (VLA_STAGE_* in vla_prefix.h)
 STAGES = ("rowstat", "gemm_qkv", "attn_prefill", "gemm_o", "gemm_gateup", "gemm_down", "kv_len",
-          "dec_qkv", "dec_attn", "dec_combine", "dec_o", "dec_gateup", "dec_down")
+          "dec_qkv", "dec_attn", "dec_o", "dec_gateup", "dec_down")
 
 STATUS = {0: "VLA_OK", 1: "VLA_ERR_INVALID_ARG", 2: "VLA_ERR_SHAPE", 3: "VLA_ERR_RANGE", 4: "VLA_ERR_KV_FULL",
           5: "VLA_ERR_NOT_PINNED", 6: "VLA_ERR_OOM", 7: "VLA_ERR_CUDA", 8: "VLA_ERR_TIMEOUT",

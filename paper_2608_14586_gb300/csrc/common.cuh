@@ -106,6 +106,18 @@ VLA_DEV void tma_load_3d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, 
         : "memory");
 }
 
+// 1-D bulk copy global -> shared (16-byte aligned addresses, size a multiple of 16), completion
+// counted in bytes on an mbarrier
+VLA_DEV void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(smem_dst)),
+                 "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
+// named barrier over `count` threads (a subset of the CTA), id 1..15
+VLA_DEV void named_sync(int id, int count) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory"); }
+
 // make this thread's generic-proxy shared-memory writes visible to the async proxy
 // (tensor core operand reads)
 VLA_DEV void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }

@@ -13,7 +13,8 @@
 //     so the weight stream starts while the input is still being staged.
 // Attention is split over the context (fixed split count -> deterministic): each CTA owns
 // one KV head (all query heads of its GQA group) and a contiguous key range, 8 lanes per key
-// row, online softmax in fp32; a combine kernel merges the partial (max, sum, output).
+// row, online softmax in fp32; the last CTA of each KV head merges the partials (max, sum,
+// output) in fixed split order.
 #include "common.cuh"
 #include "internal.h"
 
@@ -197,29 +198,63 @@ struct AttnDecParams {
     float scale_log2;
     float* part_o;   // [splits][H][dh]
     float* part_ml;  // [splits][H][2]
+    unsigned* tickets;  // [Hkv] arrival counters (0 between launches)
+    bf16* out;          // [H*dh] merged attention output
+    int cap;            // keys of one split held in shared memory (>= ceil(max_ctx / splits))
+    unsigned* status;
 };
 
-constexpr int kAttnThreads = 128;
+constexpr int kAttnThreads = 256;
+constexpr int kAttnWarps = kAttnThreads / 32;
 
+// CTA = (KV head g, split): keys [kb, ke) of the context. One thread bulk-copies the split's K
+// and V rows (contiguous in the cache) into shared memory in one round trip; the 8 warps then
+// take 2 keys per pass (16 lanes per key row, d_h/16 dims per lane) for all G query heads of
+// the group with an fp32 online softmax; warp states merge in shared memory into the split's
+// partial (max, sum, unnormalised output). The last CTA of the KV head to finish (atomic
+// ticket) merges the splits in fixed order and writes the attention output.
 template <int DH, int G>
-__global__ void __launch_bounds__(kAttnThreads) attn_decode_partial_kernel(AttnDecParams p) {
-    constexpr int DPL = DH / 8;  // dims per lane (8 lanes per key row)
-    constexpr int NW = kAttnThreads / 32;
-    __shared__ float sm_m[NW][G], sm_l[NW][G];
-    __shared__ float sm_o[NW][G][DH];
+__global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams p) {
+    constexpr int DPL = DH / 16;
+    extern __shared__ __align__(128) uint8_t smem[];
+    bf16* sK = reinterpret_cast<bf16*>(smem);
+    bf16* sV = sK + (size_t)p.cap * DH;
+    float* scratch = reinterpret_cast<float*>(sV + (size_t)p.cap * DH);
+    __shared__ uint64_t bar;
+    __shared__ float sm_m[kAttnWarps][G], sm_l[kAttnWarps][G];
+    __shared__ float sm_o[kAttnWarps][G][DH];
+    __shared__ unsigned s_ticket;
+    __shared__ int s_ok;
     const int kvh = blockIdx.x, split = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int sub = lane >> 3, l8 = lane & 7;
+    const int sub = lane >> 4, l16 = lane & 15;
     const int ctx = *p.d_len + 1;
     const int chunk = (ctx + p.splits - 1) / p.splits;
     const int kb = split * chunk;
     const int ke = min(ctx, kb + chunk);
-
+    const int nk = max(0, min(ke - kb, p.cap));
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+        s_ok = 1;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const uint32_t bytes = (uint32_t)nk * DH * 2u;
+        mbar_arrive_expect_tx(&bar, 2u * bytes);
+        if (bytes) {
+            const size_t off = ((size_t)kvh * p.max_ctx + kb) * DH;
+            bulk_load(sK, p.kc + off, bytes, &bar);
+            bulk_load(sV, p.vc + off, bytes, &bar);
+        }
+    }
     float qv[G][DPL];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh)
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) qv[hh][d] = p.q[(kvh * G + hh) * DH + l8 * DPL + d] * p.scale_log2;
+        for (int d = 0; d < DPL; ++d) qv[hh][d] = p.q[(kvh * G + hh) * DH + l16 * DPL + d] * p.scale_log2;
+    if (!mbar_wait(&bar, 0)) s_ok = 0;  // bounded; the copy itself always completes
+    __syncthreads();
     float m[G], l[G], o[G][DPL];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
@@ -228,95 +263,81 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_partial_kernel(AttnD
 #pragma unroll
         for (int d = 0; d < DPL; ++d) o[hh][d] = 0.f;
     }
-    const bf16* kbase = p.kc + (size_t)kvh * p.max_ctx * DH + l8 * DPL;
-    const bf16* vbase = p.vc + (size_t)kvh * p.max_ctx * DH + l8 * DPL;
-    // The loop bound is warp-uniform (k0 steps by warp); each 8-lane slot takes key k0 + sub
-    // and skips the update when that key is past the range, so every lane reaches every
-    // full-warp shuffle below.
-    for (int k0 = kb + warp * 4; k0 < ke; k0 += NW * 4) {
-        const int k = k0 + sub;
-        const bool valid = k < ke;
-        uint4 kr[DPL / 8], vr[DPL / 8];
+    if (s_ok) {
+        for (int k0 = warp * 2; k0 < nk; k0 += kAttnWarps * 2) {  // warp-uniform bound
+            const int k = k0 + sub;
+            const bool valid = k < nk;
+            float kf[DPL], vf[DPL];
+            const bf16* kr = sK + (size_t)(valid ? k : 0) * DH + l16 * DPL;
+            const bf16* vr = sV + (size_t)(valid ? k : 0) * DH + l16 * DPL;
 #pragma unroll
-        for (int c = 0; c < DPL / 8; ++c) {
-            if (valid) {
-                kr[c] = ldg_stream(kbase + (size_t)k * DH + c * 8);
-                vr[c] = ldg_stream(vbase + (size_t)k * DH + c * 8);
-            } else {
-                kr[c] = make_uint4(0u, 0u, 0u, 0u);
-                vr[c] = make_uint4(0u, 0u, 0u, 0u);
+            for (int c = 0; c < DPL / 4; ++c) {
+                const uint2 kw = *reinterpret_cast<const uint2*>(kr + 4 * c);
+                const uint2 vw = *reinterpret_cast<const uint2*>(vr + 4 * c);
+                kf[4 * c] = bf16_lo(kw.x);
+                kf[4 * c + 1] = bf16_hi(kw.x);
+                kf[4 * c + 2] = bf16_lo(kw.y);
+                kf[4 * c + 3] = bf16_hi(kw.y);
+                vf[4 * c] = bf16_lo(vw.x);
+                vf[4 * c + 1] = bf16_hi(vw.x);
+                vf[4 * c + 2] = bf16_lo(vw.y);
+                vf[4 * c + 3] = bf16_hi(vw.y);
             }
-        }
-        float kf[DPL], vf[DPL];
 #pragma unroll
-        for (int c = 0; c < DPL / 8; ++c) {
-            const uint32_t kw[4] = {kr[c].x, kr[c].y, kr[c].z, kr[c].w};
-            const uint32_t vw[4] = {vr[c].x, vr[c].y, vr[c].z, vr[c].w};
+            for (int hh = 0; hh < G; ++hh) {
+                float sc = 0.f;
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                kf[c * 8 + 2 * i] = bf16_lo(kw[i]);
-                kf[c * 8 + 2 * i + 1] = bf16_hi(kw[i]);
-                vf[c * 8 + 2 * i] = bf16_lo(vw[i]);
-                vf[c * 8 + 2 * i + 1] = bf16_hi(vw[i]);
+                for (int d = 0; d < DPL; ++d) sc = fmaf(qv[hh][d], kf[d], sc);
+                sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 1);
+                sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 2);
+                sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 4);
+                sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 8);
+                if (!valid) continue;
+                const float mn = fmaxf(m[hh], sc);
+                const float c = exp2f(m[hh] - mn);
+                const float pe = exp2f(sc - mn);
+                l[hh] = l[hh] * c + pe;
+#pragma unroll
+                for (int d = 0; d < DPL; ++d) o[hh][d] = fmaf(o[hh][d], c, pe * vf[d]);
+                m[hh] = mn;
             }
-        }
-#pragma unroll
-        for (int hh = 0; hh < G; ++hh) {
-            float s = 0.f;
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) s = fmaf(qv[hh][d], kf[d], s);
-            s += __shfl_xor_sync(0xFFFFFFFFu, s, 1);
-            s += __shfl_xor_sync(0xFFFFFFFFu, s, 2);
-            s += __shfl_xor_sync(0xFFFFFFFFu, s, 4);
-            if (!valid) continue;
-            const float mn = fmaxf(m[hh], s);
-            const float c = exp2f(m[hh] - mn);  // m = -inf -> 0
-            const float pe = exp2f(s - mn);
-            l[hh] = l[hh] * c + pe;
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) o[hh][d] = fmaf(o[hh][d], c, pe * vf[d]);
-            m[hh] = mn;
         }
     }
-    // merge the 4 key slots of the warp (lanes l8, l8+8, l8+16, l8+24)
+    // merge the two key slots of the warp (lanes l16 and l16 + 16), then the warps
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
+        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m[hh], 16);
+        const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l[hh], 16);
+        const float mn = fmaxf(m[hh], m2);
+        const float c1 = (mn == -INFINITY) ? 0.f : exp2f(m[hh] - mn);
+        const float c2 = (mn == -INFINITY) ? 0.f : exp2f(m2 - mn);
+        l[hh] = l[hh] * c1 + l2 * c2;
 #pragma unroll
-        for (int off = 8; off <= 16; off <<= 1) {
-            const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m[hh], off);
-            const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l[hh], off);
-            const float mn = fmaxf(m[hh], m2);
-            const float c1 = (mn == -INFINITY) ? 0.f : exp2f(m[hh] - mn);
-            const float c2 = (mn == -INFINITY) ? 0.f : exp2f(m2 - mn);
-            l[hh] = l[hh] * c1 + l2 * c2;
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) {
-                const float o2 = __shfl_xor_sync(0xFFFFFFFFu, o[hh][d], off);
-                o[hh][d] = o[hh][d] * c1 + o2 * c2;
-            }
-            m[hh] = mn;
+        for (int d = 0; d < DPL; ++d) {
+            const float o2 = __shfl_xor_sync(0xFFFFFFFFu, o[hh][d], 16);
+            o[hh][d] = o[hh][d] * c1 + o2 * c2;
         }
+        m[hh] = mn;
     }
     if (sub == 0) {
 #pragma unroll
         for (int hh = 0; hh < G; ++hh) {
-            if (l8 == 0) {
+            if (l16 == 0) {
                 sm_m[warp][hh] = m[hh];
                 sm_l[warp][hh] = l[hh];
             }
 #pragma unroll
-            for (int d = 0; d < DPL; ++d) sm_o[warp][hh][l8 * DPL + d] = o[hh][d];
+            for (int d = 0; d < DPL; ++d) sm_o[warp][hh][l16 * DPL + d] = o[hh][d];
         }
     }
     __syncthreads();
-    // merge warps: thread t handles (head hh, dim d) entries
     for (int e = threadIdx.x; e < G * DH; e += kAttnThreads) {
         const int hh = e / DH, d = e % DH;
         float mx = -INFINITY;
-        for (int w = 0; w < NW; ++w) mx = fmaxf(mx, sm_m[w][hh]);
+        for (int w = 0; w < kAttnWarps; ++w) mx = fmaxf(mx, sm_m[w][hh]);
         float lt = 0.f, ot = 0.f;
         if (mx != -INFINITY) {
-            for (int w = 0; w < NW; ++w) {
+            for (int w = 0; w < kAttnWarps; ++w) {
                 const float c = exp2f(sm_m[w][hh] - mx);
                 lt += sm_l[w][hh] * c;
                 ot += sm_o[w][hh][d] * c;
@@ -329,25 +350,48 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_partial_kernel(AttnD
             p.part_ml[((size_t)split * p.H + h) * 2 + 1] = lt;
         }
     }
-}
-
-// out[h*dh + d] = sum_s o_s e^(m_s - M) / sum_s l_s e^(m_s - M)   (fixed split order)
-__global__ void attn_decode_combine_kernel(const float* part_o, const float* part_ml, int H, int dh, int splits,
-                                           bf16* out) {
-    const int h = blockIdx.x;
-    for (int d = threadIdx.x; d < dh; d += blockDim.x) {
-        float mx = -INFINITY;
-        for (int s = 0; s < splits; ++s) mx = fmaxf(mx, part_ml[((size_t)s * H + h) * 2]);
-        float lt = 0.f, ot = 0.f;
-        for (int s = 0; s < splits; ++s) {
-            const float ms = part_ml[((size_t)s * H + h) * 2];
-            if (ms == -INFINITY) continue;
-            const float c = exp2f(ms - mx);
-            lt += part_ml[((size_t)s * H + h) * 2 + 1] * c;
-            ot += part_o[((size_t)s * H + h) * dh + d] * c;
-        }
-        out[h * dh + d] = __float2bfloat16_rn(ot / lt);
+    if (!s_ok && threadIdx.x == 0) set_status(p.status, kDevTimeout);
+    // the last CTA of this KV head merges its splits (fixed order), then re-arms the counter
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_ticket = atomicAdd(&p.tickets[kvh], 1u);
+    __syncthreads();
+    if (s_ticket != (unsigned)(p.splits - 1)) return;
+    __threadfence();
+    float* wgt = scratch;                   // [G][splits] max -> weights
+    float* wl = scratch + G * p.splits;     // [G][splits] sums
+    float* tot = wl + G * p.splits;         // [G]
+    for (int e = threadIdx.x; e < G * p.splits; e += kAttnThreads) {
+        const int hh = e / p.splits, s2 = e % p.splits;
+        const float2 ml = __ldcg(reinterpret_cast<const float2*>(p.part_ml + ((size_t)s2 * p.H + kvh * G + hh) * 2));
+        wgt[e] = ml.x;
+        wl[e] = ml.y;
     }
+    __syncthreads();
+    if (threadIdx.x < G) {
+        const int hh = threadIdx.x;
+        float mx = -INFINITY;
+        for (int s2 = 0; s2 < p.splits; ++s2) mx = fmaxf(mx, wgt[hh * p.splits + s2]);
+        float lt = 0.f;
+        for (int s2 = 0; s2 < p.splits; ++s2) {
+            const float ms = wgt[hh * p.splits + s2];
+            const float c = (ms == -INFINITY) ? 0.f : exp2f(ms - mx);
+            wgt[hh * p.splits + s2] = c;
+            lt += wl[hh * p.splits + s2] * c;
+        }
+        tot[hh] = lt;
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < G * DH; e += kAttnThreads) {
+        const int hh = e / DH, d = e % DH;
+        const int h = kvh * G + hh;
+        float ot = 0.f;
+#pragma unroll 16
+        for (int s2 = 0; s2 < p.splits; ++s2)
+            ot += __ldcg(p.part_o + ((size_t)s2 * p.H + h) * DH + d) * wgt[hh * p.splits + s2];
+        p.out[h * DH + d] = __float2bfloat16_rn(ot / tot[hh]);
+    }
+    if (threadIdx.x == 0) p.tickets[kvh] = 0u;
 }
 
 __global__ void advance_lengths_kernel(int* d_len, int count) {
@@ -374,7 +418,15 @@ cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s) {
 
 template <int DH, int G>
 cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s) {
-    attn_decode_partial_kernel<DH, G><<<dim3(p.Hkv, p.splits), kAttnThreads, 0, s>>>(p);
+    const size_t smem = (size_t)2 * p.cap * DH * 2 + (size_t)(2 * G * p.splits + G) * sizeof(float);
+    static size_t attr = 0;
+    if (smem > attr) {
+        cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        attr = smem;
+    }
+    attn_decode_kernel<DH, G><<<dim3(p.Hkv, p.splits), kAttnThreads, smem, s>>>(p);
     return cudaGetLastError();
 }
 
@@ -436,14 +488,13 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)d.dh);
     a.part_o = w.part_o;
     a.part_ml = w.part_ml;
+    a.tickets = w.tickets;
+    a.out = w.attn;
+    a.cap = (d.max_ctx + w.splits - 1) / w.splits;
+    a.status = w.status;
     hook(kStageDecAttn, true);
     e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, stream);
     hook(kStageDecAttn, false);
-    if (e != cudaSuccess) return e;
-    hook(kStageDecCombine, true);
-    attn_decode_combine_kernel<<<d.H, d.dh, 0, stream>>>(w.part_o, w.part_ml, d.H, d.dh, w.splits, w.attn);
-    e = cudaGetLastError();
-    hook(kStageDecCombine, false);
     if (e != cudaSuccess) return e;
     // 3. O projection + residual
     GemvParams o = {};

@@ -111,6 +111,7 @@ struct DecodeWork {
     bf16* m;           // [F_pad]
     const float2* rope;
     unsigned* status;
+    unsigned* tickets;  // [Hkv] split-merge counters, zero between launches
     int splits;
 };
 // Optional per-launch hook (measurement): called with (ctx, stage, begin) around each kernel.
@@ -123,8 +124,7 @@ struct StageHook {
 };
 
 // Stage ids of the decode kernels (match VLA_STAGE_DEC_* in vla_prefix.h)
-enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecCombine = 9, kStageDecO = 10, kStageDecGateUp = 11,
-             kStageDecDown = 12 };
+enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecO = 9, kStageDecGateUp = 10, kStageDecDown = 11 };
 
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
                                 bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook);
