@@ -251,6 +251,20 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) {
 // ----------------------------------------------------------------------------------------
 // Programmatic dependent launch
 // ----------------------------------------------------------------------------------------
+// Thread-block cluster: barrier over all threads of all CTAs of the cluster (release/acquire
+// orders shared-memory writes before it with distributed-shared-memory reads after it), and a
+// 32-bit load from the same shared-memory variable in CTA `rank` of the cluster.
+VLA_DEV void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+VLA_DEV float ld_dsmem_f32(const float* local, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+    return v;
+}
+
 VLA_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 VLA_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

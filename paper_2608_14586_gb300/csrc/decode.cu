@@ -9,12 +9,15 @@
 //     SwiGLU, consecutive rows for the residual projections;
 //   * the input vector is staged in shared memory; RMSNorm's 1/rms is computed per CTA
 //     (the gains are folded into the weights);
-//   * each kernel prefetches its first weight rows into L2 before reading its input vector,
-//     so the weight stream starts while the input is still being staged.
-// Attention is split over the context (fixed split count -> deterministic): each CTA owns
-// one KV head (all query heads of its GQA group) and a contiguous key range, 8 lanes per key
-// row, online softmax in fp32; the last CTA of each KV head merges the partials (max, sum,
-// output) in fixed split order.
+//   * under programmatic dependent launch each kernel starts while its predecessor drains:
+//     it prefetches its first weight rows into L2 and loads the first batch into registers,
+//     and reads nothing that an earlier kernel of the step wrote before griddepcontrol.wait.
+// Attention is split over the context inside one thread-block cluster per KV head (16 CTAs
+// where the device schedules such clusters, else 8; fixed split count -> deterministic): each
+// CTA bulk-copies its contiguous key range of K and V into shared memory (the rows that
+// predate the step before the wait, so the copy overlaps the QKV kernel), scores it for all
+// query heads of the GQA group with an online softmax, and the cluster merges the partial
+// (max, sum, output) states through distributed shared memory in fixed rank order.
 #include "common.cuh"
 #include "internal.h"
 
@@ -119,7 +122,11 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
     const int nchunk = p.K >> 3;        // 16-byte chunks per row
     const int nstep = nchunk >> 5;      // chunk steps of the whole warp
 
-    // weights do not depend on the previous kernel: warm L2 with this warp's first rows
+    // Weights do not depend on the previous kernel. Under programmatic dependent launch this
+    // part runs while the previous kernel drains: warm L2 with this warp's first row pair and
+    // load its first batch of chunks into registers. Nothing written by an earlier kernel is
+    // read before pdl_wait().
+    uint4 va[kGemvU], vb[kGemvU];
     if (gw < p.units) {
         int ra, rb;
         unit_rows<MODE>(p, gw, ra, rb);
@@ -129,9 +136,20 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pa + l * 128));
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pb + l * 128));
         }
+        const uint4* wa = reinterpret_cast<const uint4*>(pa);
+        const uint4* wb = reinterpret_cast<const uint4*>(pb);
+#pragma unroll
+        for (int i = 0; i < kGemvU; ++i) {
+            if (i < nstep) {
+                va[i] = ldg_stream(wa + i * 32 + lane);
+                vb[i] = ldg_stream(wb + i * 32 + lane);
+            }
+        }
     }
+    pdl_wait();
+    pdl_trigger();
     const uint4* xg = reinterpret_cast<const uint4*>(p.xv);
-    for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) xs[i] = xg[i];
+    for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) xs[i] = __ldcg(xg + i);
     __syncthreads();
     float rinv = 1.f;
     if constexpr (MODE != kGemvResid) {
@@ -162,10 +180,9 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
         const uint4* wb = reinterpret_cast<const uint4*>(p.W + (size_t)rb * p.K);
         float acc_a = 0.f, acc_b = 0.f;
         for (int s = 0; s < nstep; s += kGemvU) {
-            uint4 va[kGemvU], vb[kGemvU];
 #pragma unroll
             for (int i = 0; i < kGemvU; ++i) {
-                if (s + i < nstep) {
+                if (s + i < nstep && (s > 0 || u != gw)) {  // batch 0 of the first unit is preloaded
                     const int c = (s + i) * 32 + lane;
                     va[i] = ldg_stream(wa + c);
                     vb[i] = ldg_stream(wb + c);
@@ -187,74 +204,97 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
 }
 
 // ---------------------------------------------------------------------------------------
-// split-KV attention
+// split-KV attention: one thread-block cluster per KV head
 // ---------------------------------------------------------------------------------------
 struct AttnDecParams {
-    const float* q;  // [H*dh]
+    const float* q;  // [H*dh] post-RoPE query, fp32
     const bf16* kc;  // layer base [Hkv][max_ctx][dh]
     const bf16* vc;
     const int* d_len;  // position of the new token; context = d_len + 1
-    int H, Hkv, max_ctx, splits;
+    int H, Hkv, max_ctx;
+    int cs;      // CTAs per cluster = key splits per KV head
+    int cap;     // keys per shared-memory stage
+    int stages;  // 1 or 2
     float scale_log2;
-    float* part_o;   // [splits][H][dh]
-    float* part_ml;  // [splits][H][2]
-    unsigned* tickets;  // [Hkv] arrival counters (0 between launches)
-    bf16* out;          // [H*dh] merged attention output
-    int cap;            // keys of one split held in shared memory (>= ceil(max_ctx / splits))
+    bf16* out;  // [H*dh] attention output
     unsigned* status;
 };
 
 constexpr int kAttnThreads = 256;
 constexpr int kAttnWarps = kAttnThreads / 32;
+constexpr int kMaxCluster = 16;
 
-// CTA = (KV head g, split): keys [kb, ke) of the context. One thread bulk-copies the split's K
-// and V rows (contiguous in the cache) into shared memory in one round trip; the 8 warps then
-// take 2 keys per pass (16 lanes per key row, d_h/16 dims per lane) for all G query heads of
-// the group with an fp32 online softmax; warp states merge in shared memory into the split's
-// partial (max, sum, unnormalised output). The last CTA of the KV head to finish (atomic
-// ticket) merges the splits in fixed order and writes the attention output.
+template <int DPL>
+VLA_DEV void load_row_part(const bf16* src, float (&f)[DPL]) {
+    if constexpr (DPL == 8) {
+        const uint4 w = *reinterpret_cast<const uint4*>(src);
+        f[0] = bf16_lo(w.x), f[1] = bf16_hi(w.x), f[2] = bf16_lo(w.y), f[3] = bf16_hi(w.y);
+        f[4] = bf16_lo(w.z), f[5] = bf16_hi(w.z), f[6] = bf16_lo(w.w), f[7] = bf16_hi(w.w);
+    } else {
+        const uint2 w = *reinterpret_cast<const uint2*>(src);
+        f[0] = bf16_lo(w.x), f[1] = bf16_hi(w.x), f[2] = bf16_lo(w.y), f[3] = bf16_hi(w.y);
+    }
+}
+
+// Cluster (cs CTAs) = KV head g; CTA rank r owns keys [r*ceil(ctx/cs), ...) of the context.
+// Thread 0 bulk-copies the rows of each chunk (cap keys) of K and V into a shared-memory stage;
+// 8 warps take 2 keys per pass (16 lanes per key row, d_h/16 dims per lane) for all G query
+// heads of the group with an fp32 online softmax (scores in the log2 domain). Warp states merge
+// in shared memory into the CTA's (max, sum, unnormalised output); after a cluster barrier, CTA
+// r merges output elements [r*G*dh/cs, (r+1)*G*dh/cs) over the cs CTAs through distributed
+// shared memory, in fixed rank order, and writes them. No partials leave the chip.
 template <int DH, int G>
 __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams p) {
     constexpr int DPL = DH / 16;
     extern __shared__ __align__(128) uint8_t smem[];
-    bf16* sK = reinterpret_cast<bf16*>(smem);
-    bf16* sV = sK + (size_t)p.cap * DH;
-    float* scratch = reinterpret_cast<float*>(sV + (size_t)p.cap * DH);
-    __shared__ uint64_t bar;
+    __shared__ uint64_t full[2];
     __shared__ float sm_m[kAttnWarps][G], sm_l[kAttnWarps][G];
     __shared__ float sm_o[kAttnWarps][G][DH];
-    __shared__ unsigned s_ticket;
+    __shared__ float c_m[G], c_l[G];
+    __shared__ __align__(16) float c_o[G * DH];
     __shared__ int s_ok;
-    const int kvh = blockIdx.x, split = blockIdx.y;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rank = blockIdx.x, kvh = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int sub = lane >> 4, l16 = lane & 15;
+    const size_t stage_elems = (size_t)2 * p.cap * DH;  // K rows then V rows
+    bf16* const sbase = reinterpret_cast<bf16*>(smem);
+    // d_len was last written by an earlier step (complete before this one started)
     const int ctx = *p.d_len + 1;
-    const int chunk = (ctx + p.splits - 1) / p.splits;
-    const int kb = split * chunk;
-    const int ke = min(ctx, kb + chunk);
-    const int nk = max(0, min(ke - kb, p.cap));
-    if (threadIdx.x == 0) {
-        mbar_init(&bar, 1);
+    const int per = (ctx + p.cs - 1) / p.cs;
+    const int kb = rank * per;
+    const int ke = min(ctx, kb + per);
+    const int nk = max(0, ke - kb);
+    const int nchunks = (nk + p.cap - 1) / p.cap;
+    const int new_row = ctx - 1;  // written by the QKV kernel this one depends on
+    // bulk copy of chunk c's rows that existed before this step (rows < new_row)
+    auto issue = [&](int c) {
+        const int r0 = kb + c * p.cap;
+        const int rows = min(p.cap, ke - r0);
+        const int old_rows = max(0, min(rows, new_row - r0));
+        const uint32_t bytes = (uint32_t)old_rows * DH * 2u;
+        bf16* sk = sbase + (size_t)(c % p.stages) * stage_elems;
+        uint64_t* bar = &full[c % p.stages];
+        mbar_arrive_expect_tx(bar, 2u * bytes);
+        if (bytes) {
+            const size_t off = ((size_t)kvh * p.max_ctx + r0) * DH;
+            bulk_load(sk, p.kc + off, bytes, bar);
+            bulk_load(sk + (size_t)p.cap * DH, p.vc + off, bytes, bar);
+        }
+    };
+    if (tid == 0) {
+        mbar_init(&full[0], 1);
+        mbar_init(&full[1], 1);
         fence_barrier_init();
         s_ok = 1;
+        for (int c = 0; c < min(nchunks, p.stages); ++c) issue(c);
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        const uint32_t bytes = (uint32_t)nk * DH * 2u;
-        mbar_arrive_expect_tx(&bar, 2u * bytes);
-        if (bytes) {
-            const size_t off = ((size_t)kvh * p.max_ctx + kb) * DH;
-            bulk_load(sK, p.kc + off, bytes, &bar);
-            bulk_load(sV, p.vc + off, bytes, &bar);
-        }
-    }
+    pdl_wait();
+    pdl_trigger();
     float qv[G][DPL];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh)
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) qv[hh][d] = p.q[(kvh * G + hh) * DH + l16 * DPL + d] * p.scale_log2;
-    if (!mbar_wait(&bar, 0)) s_ok = 0;  // bounded; the copy itself always completes
-    __syncthreads();
+        for (int d = 0; d < DPL; ++d) qv[hh][d] = __ldcg(p.q + (kvh * G + hh) * DH + l16 * DPL + d) * p.scale_log2;
     float m[G], l[G], o[G][DPL];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
@@ -263,26 +303,29 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
 #pragma unroll
         for (int d = 0; d < DPL; ++d) o[hh][d] = 0.f;
     }
-    if (s_ok) {
-        for (int k0 = warp * 2; k0 < nk; k0 += kAttnWarps * 2) {  // warp-uniform bound
+    __syncthreads();  // barrier init visible before any wait
+    for (int c = 0; c < nchunks; ++c) {
+        const int r0 = kb + c * p.cap;
+        const int rows = min(p.cap, ke - r0);
+        const bf16* sk = sbase + (size_t)(c % p.stages) * stage_elems;
+        const bf16* sv = sk + (size_t)p.cap * DH;
+        const int nr = new_row - r0;
+        if (nr >= 0 && nr < rows && tid < DH / 8) {
+            const size_t off = ((size_t)kvh * p.max_ctx + new_row) * DH;
+            reinterpret_cast<uint4*>(const_cast<bf16*>(sk) + (size_t)nr * DH)[tid] =
+                __ldcg(reinterpret_cast<const uint4*>(p.kc + off) + tid);
+            reinterpret_cast<uint4*>(const_cast<bf16*>(sv) + (size_t)nr * DH)[tid] =
+                __ldcg(reinterpret_cast<const uint4*>(p.vc + off) + tid);
+        }
+        if (!mbar_wait(&full[c % p.stages], (uint32_t)(c / p.stages) & 1u)) s_ok = 0;
+        __syncthreads();
+        if (!s_ok) break;  // CTA-uniform
+        for (int k0 = warp * 2; k0 < rows; k0 += kAttnWarps * 2) {  // warp-uniform bound
             const int k = k0 + sub;
-            const bool valid = k < nk;
+            const bool valid = k < rows;
             float kf[DPL], vf[DPL];
-            const bf16* kr = sK + (size_t)(valid ? k : 0) * DH + l16 * DPL;
-            const bf16* vr = sV + (size_t)(valid ? k : 0) * DH + l16 * DPL;
-#pragma unroll
-            for (int c = 0; c < DPL / 4; ++c) {
-                const uint2 kw = *reinterpret_cast<const uint2*>(kr + 4 * c);
-                const uint2 vw = *reinterpret_cast<const uint2*>(vr + 4 * c);
-                kf[4 * c] = bf16_lo(kw.x);
-                kf[4 * c + 1] = bf16_hi(kw.x);
-                kf[4 * c + 2] = bf16_lo(kw.y);
-                kf[4 * c + 3] = bf16_hi(kw.y);
-                vf[4 * c] = bf16_lo(vw.x);
-                vf[4 * c + 1] = bf16_hi(vw.x);
-                vf[4 * c + 2] = bf16_lo(vw.y);
-                vf[4 * c + 3] = bf16_hi(vw.y);
-            }
+            load_row_part<DPL>(sk + (size_t)(valid ? k : 0) * DH + l16 * DPL, kf);
+            load_row_part<DPL>(sv + (size_t)(valid ? k : 0) * DH + l16 * DPL, vf);
 #pragma unroll
             for (int hh = 0; hh < G; ++hh) {
                 float sc = 0.f;
@@ -292,25 +335,28 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
                 sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 2);
                 sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 4);
                 sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 8);
-                if (!valid) continue;
-                const float mn = fmaxf(m[hh], sc);
-                const float c = exp2f(m[hh] - mn);
-                const float pe = exp2f(sc - mn);
-                l[hh] = l[hh] * c + pe;
+                if (valid) {
+                    const float mn = fmaxf(m[hh], sc);
+                    const float cr = ex2_approx(m[hh] - mn);
+                    const float pe = ex2_approx(sc - mn);
+                    l[hh] = fmaf(l[hh], cr, pe);
 #pragma unroll
-                for (int d = 0; d < DPL; ++d) o[hh][d] = fmaf(o[hh][d], c, pe * vf[d]);
-                m[hh] = mn;
+                    for (int d = 0; d < DPL; ++d) o[hh][d] = fmaf(o[hh][d], cr, pe * vf[d]);
+                    m[hh] = mn;
+                }
             }
         }
+        __syncthreads();  // stage free
+        if (tid == 0 && c + p.stages < nchunks) issue(c + p.stages);
     }
-    // merge the two key slots of the warp (lanes l16 and l16 + 16), then the warps
+    // merge the two key slots of each warp (lanes l16 and l16 + 16), then the warps
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
         const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m[hh], 16);
         const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l[hh], 16);
         const float mn = fmaxf(m[hh], m2);
-        const float c1 = (mn == -INFINITY) ? 0.f : exp2f(m[hh] - mn);
-        const float c2 = (mn == -INFINITY) ? 0.f : exp2f(m2 - mn);
+        const float c1 = (mn == -INFINITY) ? 0.f : ex2_approx(m[hh] - mn);
+        const float c2 = (mn == -INFINITY) ? 0.f : ex2_approx(m2 - mn);
         l[hh] = l[hh] * c1 + l2 * c2;
 #pragma unroll
         for (int d = 0; d < DPL; ++d) {
@@ -331,67 +377,57 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
         }
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < G * DH; e += kAttnThreads) {
+    for (int e = tid; e < G * DH; e += kAttnThreads) {
         const int hh = e / DH, d = e % DH;
         float mx = -INFINITY;
+#pragma unroll
         for (int w = 0; w < kAttnWarps; ++w) mx = fmaxf(mx, sm_m[w][hh]);
         float lt = 0.f, ot = 0.f;
         if (mx != -INFINITY) {
+#pragma unroll
             for (int w = 0; w < kAttnWarps; ++w) {
-                const float c = exp2f(sm_m[w][hh] - mx);
-                lt += sm_l[w][hh] * c;
-                ot += sm_o[w][hh][d] * c;
+                const float cw = ex2_approx(sm_m[w][hh] - mx);
+                lt = fmaf(sm_l[w][hh], cw, lt);
+                ot = fmaf(sm_o[w][hh][d], cw, ot);
             }
         }
-        const int h = kvh * G + hh;
-        p.part_o[((size_t)split * p.H + h) * DH + d] = ot;
+        c_o[e] = ot;
         if (d == 0) {
-            p.part_ml[((size_t)split * p.H + h) * 2 + 0] = mx;
-            p.part_ml[((size_t)split * p.H + h) * 2 + 1] = lt;
+            c_m[hh] = mx;
+            c_l[hh] = lt;
         }
     }
-    if (!s_ok && threadIdx.x == 0) set_status(p.status, kDevTimeout);
-    // the last CTA of this KV head merges its splits (fixed order), then re-arms the counter
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) s_ticket = atomicAdd(&p.tickets[kvh], 1u);
-    __syncthreads();
-    if (s_ticket != (unsigned)(p.splits - 1)) return;
-    __threadfence();
-    float* wgt = scratch;                   // [G][splits] max -> weights
-    float* wl = scratch + G * p.splits;     // [G][splits] sums
-    float* tot = wl + G * p.splits;         // [G]
-    for (int e = threadIdx.x; e < G * p.splits; e += kAttnThreads) {
-        const int hh = e / p.splits, s2 = e % p.splits;
-        const float2 ml = __ldcg(reinterpret_cast<const float2*>(p.part_ml + ((size_t)s2 * p.H + kvh * G + hh) * 2));
-        wgt[e] = ml.x;
-        wl[e] = ml.y;
-    }
-    __syncthreads();
-    if (threadIdx.x < G) {
-        const int hh = threadIdx.x;
+    if (!s_ok && tid == 0) set_status(p.status, kDevTimeout);
+    cluster_sync_all();  // every CTA's (c_m, c_l, c_o) is complete and visible to the cluster
+    const int per_cta = G * DH / p.cs;
+    if (tid < per_cta) {
+        const int e = rank * per_cta + tid;
+        const int hh = e / DH;
+        float mr[kMaxCluster], lr[kMaxCluster], orr[kMaxCluster];
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r) {
+            if (r < p.cs) {
+                mr[r] = ld_dsmem_f32(&c_m[hh], (uint32_t)r);
+                lr[r] = ld_dsmem_f32(&c_l[hh], (uint32_t)r);
+                orr[r] = ld_dsmem_f32(&c_o[e], (uint32_t)r);
+            }
+        }
         float mx = -INFINITY;
-        for (int s2 = 0; s2 < p.splits; ++s2) mx = fmaxf(mx, wgt[hh * p.splits + s2]);
-        float lt = 0.f;
-        for (int s2 = 0; s2 < p.splits; ++s2) {
-            const float ms = wgt[hh * p.splits + s2];
-            const float c = (ms == -INFINITY) ? 0.f : exp2f(ms - mx);
-            wgt[hh * p.splits + s2] = c;
-            lt += wl[hh * p.splits + s2] * c;
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r)
+            if (r < p.cs) mx = fmaxf(mx, mr[r]);
+        float lt = 0.f, ot = 0.f;
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r) {
+            if (r < p.cs && mr[r] != -INFINITY) {
+                const float cw = ex2_approx(mr[r] - mx);
+                lt = fmaf(lr[r], cw, lt);
+                ot = fmaf(orr[r], cw, ot);
+            }
         }
-        tot[hh] = lt;
+        p.out[kvh * G * DH + e] = __float2bfloat16_rn(ot / lt);
     }
-    __syncthreads();
-    for (int e = threadIdx.x; e < G * DH; e += kAttnThreads) {
-        const int hh = e / DH, d = e % DH;
-        const int h = kvh * G + hh;
-        float ot = 0.f;
-#pragma unroll 16
-        for (int s2 = 0; s2 < p.splits; ++s2)
-            ot += __ldcg(p.part_o + ((size_t)s2 * p.H + h) * DH + d) * wgt[hh * p.splits + s2];
-        p.out[h * DH + d] = __float2bfloat16_rn(ot / tot[hh]);
-    }
-    if (threadIdx.x == 0) p.tickets[kvh] = 0u;
+    cluster_sync_all();  // keep this CTA's shared memory alive until the cluster has read it
 }
 
 __global__ void advance_lengths_kernel(int* d_len, int count) {
@@ -399,8 +435,26 @@ __global__ void advance_lengths_kernel(int* d_len, int count) {
     if (i < count) d_len[i] += 1;
 }
 
+// Launch with programmatic stream serialization when `pdl` is set: the kernel may start while
+// the previous kernel in the stream drains; every decode kernel reads data produced by its
+// predecessors only after griddepcontrol.wait and writes nothing before it.
+template <typename Kern, typename... Args>
+cudaError_t launch_kernel(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 template <int MODE>
-cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s) {
+cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
     const size_t smem = (size_t)p.K * 2;
     static bool attr_set = false;
     if (!attr_set) {
@@ -412,48 +466,134 @@ cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s) {
     int grid = 2 * num_sms;
     const int gmax = (warps_needed + 7) / 8;
     if (grid > gmax) grid = gmax;
-    gemv_kernel<MODE><<<grid, kGemvThreads, smem, s>>>(p);
-    return cudaGetLastError();
+    return launch_kernel(gemv_kernel<MODE>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
 }
 
 template <int DH, int G>
-cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s) {
-    const size_t smem = (size_t)2 * p.cap * DH * 2 + (size_t)(2 * G * p.splits + G) * sizeof(float);
-    static size_t attr = 0;
-    if (smem > attr) {
-        cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
-        if (e != cudaSuccess) return e;
-        attr = smem;
-    }
-    attn_decode_kernel<DH, G><<<dim3(p.Hkv, p.splits), kAttnThreads, smem, s>>>(p);
-    return cudaGetLastError();
+size_t attn_dec_smem(const AttnDecParams& p) {
+    return (size_t)p.stages * 2 * p.cap * DH * sizeof(bf16);
 }
 
-cudaError_t launch_attn_dec_any(int dh, int group, const AttnDecParams& p, cudaStream_t s) {
-    if (dh == 128) {
-        switch (group) {
-            case 1: return launch_attn_dec<128, 1>(p, s);
-            case 2: return launch_attn_dec<128, 2>(p, s);
-            case 4: return launch_attn_dec<128, 4>(p, s);
-            case 8: return launch_attn_dec<128, 8>(p, s);
+template <int DH, int G>
+cudaError_t attn_dec_prepare(int cs, size_t smem) {
+    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<DH, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e == cudaSuccess && cs > 8)
+        e = cudaFuncSetAttribute(attn_decode_kernel<DH, G>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+}
+
+template <int DH, int G>
+cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s, bool pdl) {
+    const size_t smem = attn_dec_smem<DH, G>(p);
+    static size_t attr_smem = 0;
+    static int attr_cs = 0;
+    if (smem > attr_smem || p.cs > attr_cs) {
+        cudaError_t e = attn_dec_prepare<DH, G>(p.cs, smem);
+        if (e != cudaSuccess) return e;
+        attr_smem = smem > attr_smem ? smem : attr_smem;
+        attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.cs, p.Hkv);
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = p.cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, attn_decode_kernel<DH, G>, p);
+}
+
+// Cluster size and shared-memory staging for a context of up to max_ctx keys: 16 CTAs per KV
+// head when the device can co-schedule such clusters, else 8; one stage holding all of a
+// CTA's keys when that fits in 160 KB, else two stages of a fixed chunk.
+template <int DH, int G>
+cudaError_t attn_dec_plan(int Hkv, int max_ctx, int* cs, int* cap, int* stages) {
+    constexpr size_t kBudget = 160 * 1024;
+    const size_t row_pair = (size_t)2 * DH * sizeof(bf16);
+    for (int c : {16, 8}) {
+        const int keys = (max_ctx + c - 1) / c;
+        int st = 1, cp = keys;
+        if ((size_t)keys * row_pair > kBudget) {
+            st = 2;
+            cp = (int)(kBudget / (2 * row_pair));
         }
-    } else if (dh == 64) {
-        switch (group) {
-            case 1: return launch_attn_dec<64, 1>(p, s);
-            case 2: return launch_attn_dec<64, 2>(p, s);
-            case 4: return launch_attn_dec<64, 4>(p, s);
-            case 8: return launch_attn_dec<64, 8>(p, s);
+        const size_t smem = (size_t)st * cp * row_pair;
+        if (attn_dec_prepare<DH, G>(c, smem) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(c, Hkv);
+        cfg.blockDim = dim3(kAttnThreads);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = c;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, attn_decode_kernel<DH, G>, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            n = 0;
+        }
+        if (n >= 1) {
+            *cs = c;
+            *cap = cp;
+            *stages = st;
+            return cudaSuccess;
         }
     }
+    return cudaErrorInvalidConfiguration;
+}
+
+#define VLA_ATTN_DISPATCH(dh, group, CALL)          \
+    if (dh == 128) {                                 \
+        switch (group) {                             \
+            case 1: return CALL(128, 1);             \
+            case 2: return CALL(128, 2);             \
+            case 4: return CALL(128, 4);             \
+            case 8: return CALL(128, 8);             \
+        }                                            \
+    } else if (dh == 64) {                           \
+        switch (group) {                             \
+            case 1: return CALL(64, 1);              \
+            case 2: return CALL(64, 2);              \
+            case 4: return CALL(64, 4);              \
+            case 8: return CALL(64, 8);              \
+        }                                            \
+    }                                                \
     return cudaErrorInvalidValue;
+
+cudaError_t launch_attn_dec_any(int dh, int group, const AttnDecParams& p, cudaStream_t s, bool pdl) {
+#define VLA_CALL(D, GG) launch_attn_dec<D, GG>(p, s, pdl)
+    VLA_ATTN_DISPATCH(dh, group, VLA_CALL)
+#undef VLA_CALL
 }
 
 }  // namespace
 
+cudaError_t plan_decode_attention(int dh, int group, int Hkv, int max_ctx, int* cs, int* cap, int* stages) {
+#define VLA_CALL(D, GG) attn_dec_plan<D, GG>(Hkv, max_ctx, cs, cap, stages)
+    VLA_ATTN_DISPATCH(dh, group, VLA_CALL)
+#undef VLA_CALL
+}
+
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
-                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook) {
+                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook, bool pdl_first) {
     cudaError_t e;
+    // stage timing records events between the launches: launch those fully serialized
+    const bool pdl = hook.fn == nullptr;
+    pdl_first = pdl_first && pdl;
     const int qc = d.H * d.dh, kvc = d.Hkv * d.dh;
     // 1. RMSNorm + QKV + RoPE + KV append
     GemvParams g = {};
@@ -472,7 +612,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     g.max_ctx = d.max_ctx;
     g.eps = d.eps;
     hook(kStageDecQKV, true);
-    e = launch_gemv<kGemvQKV>(g, num_sms, stream);
+    e = launch_gemv<kGemvQKV>(g, num_sms, stream, pdl_first);
     hook(kStageDecQKV, false);
     if (e != cudaSuccess) return e;
     // 2. split-KV attention + combine
@@ -484,16 +624,35 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     a.H = d.H;
     a.Hkv = d.Hkv;
     a.max_ctx = d.max_ctx;
-    a.splits = w.splits;
+    a.cs = w.attn_cs;
+    a.cap = w.attn_cap;
+    a.stages = w.attn_stages;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)d.dh);
-    a.part_o = w.part_o;
-    a.part_ml = w.part_ml;
-    a.tickets = w.tickets;
     a.out = w.attn;
-    a.cap = (d.max_ctx + w.splits - 1) / w.splits;
     a.status = w.status;
     hook(kStageDecAttn, true);
-    e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, stream);
+    if (w.attn_tc) {
+        CUtensorMap tk, tv;
+        if (!make_tmap_bf16_3d(&tk, L.kcache, d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32) ||
+            !make_tmap_bf16_3d(&tv, L.vcache, d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32))
+            return cudaErrorInvalidValue;
+        AttnDecTcParams t = {};
+        t.q = w.q;
+        t.kc = L.kcache;
+        t.vc = L.vcache;
+        t.d_len = L.d_len;
+        t.H = d.H;
+        t.Hkv = d.Hkv;
+        t.max_ctx = d.max_ctx;
+        t.cs = w.attn_cs;
+        t.nt = w.attn_cap;
+        t.scale_log2 = a.scale_log2;
+        t.out = w.attn;
+        t.status = w.status;
+        e = launch_attn_decode_tc(tk, tv, d.H / d.Hkv, t, stream, pdl);
+    } else {
+        e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, stream, pdl);
+    }
     hook(kStageDecAttn, false);
     if (e != cudaSuccess) return e;
     // 3. O projection + residual
@@ -505,7 +664,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     o.resid = x_in;
     o.out = w.x_mid;
     hook(kStageDecO, true);
-    e = launch_gemv<kGemvResid>(o, num_sms, stream);
+    e = launch_gemv<kGemvResid>(o, num_sms, stream, pdl);
     hook(kStageDecO, false);
     if (e != cudaSuccess) return e;
     // 4. RMSNorm + gate/up + SwiGLU
@@ -517,7 +676,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     gu.out = w.m;
     gu.eps = d.eps;
     hook(kStageDecGateUp, true);
-    e = launch_gemv<kGemvSwiGLU>(gu, num_sms, stream);
+    e = launch_gemv<kGemvSwiGLU>(gu, num_sms, stream, pdl);
     hook(kStageDecGateUp, false);
     if (e != cudaSuccess) return e;
     // 5. down projection + residual
@@ -529,7 +688,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     dn.resid = w.x_mid;
     dn.out = x_out;
     hook(kStageDecDown, true);
-    e = launch_gemv<kGemvResid>(dn, num_sms, stream);
+    e = launch_gemv<kGemvResid>(dn, num_sms, stream, pdl);
     hook(kStageDecDown, false);
     return e;
 }

@@ -1,0 +1,404 @@
+// Single-token (decode) attention on the 5th-generation tensor cores, head_dim 128.
+//
+// One thread-block cluster of `cs` CTAs per KV head g; CTA rank r owns the contiguous key range
+// [r*ceil(ctx/cs), ...) of the context (Sec. 3.2's causal attention at one query position,
+// split over keys). Per CTA, for the G query heads of the GQA group:
+//   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory.
+//      Rows that predate this step are requested before griddepcontrol.wait, so the copy
+//      overlaps the QKV kernel; the new token's row is written over its slot afterwards.
+//   2. S^T = K Q^T on tcgen05 (M = 128 keys per tile, N = 16 >= G heads, K = d_h), fp32 in TMEM.
+//   3. One thread per key row reads its G scores, the CTA takes the per-head max and sum of
+//      exp2(s * log2(e)/sqrt(d_h) - max), and writes P^T (bf16, 128-byte-swizzled K-major).
+//   4. O^T = V^T P^T on tcgen05 (M = d_h, N = 16, K = keys; V^T read MN-major in place).
+//   5. The CTA's (max, sum, unnormalised O) go to shared memory; after a cluster barrier CTA r
+//      merges output elements [r*G*d_h/cs, (r+1)*G*d_h/cs) over the cluster through
+//      distributed shared memory in fixed rank order and writes them as bf16.
+// Every mbarrier wait is bounded; a timeout sets the status word and the kernel winds down.
+#include "common.cuh"
+#include "internal.h"
+
+namespace vla {
+
+namespace {
+
+constexpr int kDH = 128;
+constexpr int kThreads = 128;
+constexpr int kBoxRows = 32;
+constexpr uint32_t kChunk = 128u * 128u;            // [128 rows][64 bf16] per d_h half
+constexpr uint32_t kTileBytes = 2u * kChunk;        // 128 keys x 128 d_h
+constexpr uint32_t kQBytes = 2u * 16u * 128u;       // [16 rows][128] as two halves of 64
+constexpr uint32_t kPTileBytes = 2u * 16u * 128u;   // [16 heads][128 keys] as two halves of 64
+constexpr uint32_t kBoxBytes = kBoxRows * 128u;     // one [32 rows][64] box
+constexpr uint32_t kTmemCols = 64;                  // S^T tiles at [16t, 16t+16), O^T at [48, 64)
+constexpr uint32_t kOCol = 48;
+constexpr int kMaxCs = 16;
+
+VLA_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+// byte offset of (row, 16-byte chunk j) inside a 128-byte-swizzled tile of 128-byte rows
+VLA_DEV uint32_t sw128_off(int row, int j) { return (uint32_t)row * 128u + ((uint32_t)(j ^ (row & 7)) << 4); }
+
+struct Smem {
+    uint32_t off_k, off_v, off_q, off_p, total;
+};
+
+__host__ __device__ inline Smem smem_layout(int nt) {
+    Smem s;
+    s.off_k = 0;
+    s.off_v = nt * kTileBytes;
+    s.off_q = 2 * nt * kTileBytes;
+    s.off_p = s.off_q + kQBytes;
+    s.total = s.off_p + nt * kPTileBytes + 1024;  // + alignment slack
+    return s;
+}
+
+template <int G>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                          AttnDecTcParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t bar_kv, bar_mma;
+    __shared__ uint32_t tmem_slot;
+    __shared__ float red_m[4][G], red_l[4][G];
+    __shared__ float c_m[G], c_l[G];
+    __shared__ __align__(16) float c_o[G * kDH];
+    __shared__ int s_ok;
+    const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
+    uint8_t* smem = smem_raw + pad;
+    const Smem L = smem_layout(p.nt);
+    uint8_t* sK = smem + L.off_k;
+    uint8_t* sV = smem + L.off_v;
+    uint8_t* sQ = smem + L.off_q;
+    uint8_t* sP = smem + L.off_p;
+    const int rank = blockIdx.x, kvh = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // d_len was last written by an earlier step (complete before this one started)
+    const int ctx = *p.d_len + 1;
+    const int per = (ctx + p.cs - 1) / p.cs;
+    const int kb = rank * per;
+    const int nk = max(0, min(min(ctx, kb + per) - kb, p.nt * 128));
+    const int nbox = (nk + kBoxRows - 1) / kBoxRows;
+    const int new_row = ctx - 1 - kb;  // slot of the token written by the QKV kernel
+
+    if (tid == 0) {
+        mbar_init(&bar_kv, 1);
+        mbar_init(&bar_mma, 1);
+        fence_barrier_init();
+        s_ok = 1;
+        tma_prefetch_desc(&tmK);
+        tma_prefetch_desc(&tmV);
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_slot, kTmemCols);
+        tmem_relinquish();
+    }
+    // zero Q rows >= G and the P^T tiles (rows >= G stay zero; rows < G are rewritten)
+    for (uint32_t i = tid; i < (kQBytes + p.nt * kPTileBytes) / 16; i += kThreads)
+        reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0u, 0u, 0u, 0u);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    if (tid == 0) {
+        mbar_arrive_expect_tx(&bar_kv, (uint32_t)nbox * 4u * kBoxBytes);
+        for (int b = 0; b < nbox; ++b) {
+            const uint32_t dst = (uint32_t)(b >> 2) * kTileBytes + (uint32_t)(b & 3) * kBoxBytes;
+            const int y = kb + b * kBoxRows;
+            for (int c = 0; c < 2; ++c) {
+                tma_load_3d(sK + dst + c * kChunk, &tmK, &bar_kv, c * 64, y, kvh);
+                tma_load_3d(sV + dst + c * kChunk, &tmV, &bar_kv, c * 64, y, kvh);
+            }
+        }
+    }
+    pdl_wait();
+    pdl_trigger();
+
+    // Q (post-RoPE, fp32) -> bf16 rows [0, G) of the swizzled K-major tile
+    for (int i = tid; i < G * 16; i += kThreads) {
+        const int hh = i >> 4, j = i & 15;  // head, 16-byte chunk of 8 dims
+        const float4* src = reinterpret_cast<const float4*>(p.q + (size_t)(kvh * G + hh) * kDH + j * 8);
+        const float4 a = __ldcg(src), b = __ldcg(src + 1);
+        *reinterpret_cast<uint4*>(sQ + (j >> 3) * (16 * 128) + sw128_off(hh, j & 7)) =
+            make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
+    }
+    if (!mbar_wait(&bar_kv, 0)) s_ok = 0;
+    // the new token's K and V rows over their (stale) slots; V rows past the range -> 0 so that
+    // zero probabilities never meet non-finite values
+    if (new_row >= 0 && new_row < nk && tid < 32) {
+        const int half = tid >> 4, j = (tid >> 1) & 7, which = tid & 1;  // 2 halves x 8 chunks x {K, V}
+        const bf16* src = (which ? p.vc : p.kc) + ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + half * 64 + j * 8;
+        uint8_t* dst = (which ? sV : sK) + (uint32_t)(new_row >> 7) * kTileBytes + half * kChunk +
+                       sw128_off(new_row & 127, j);
+        *reinterpret_cast<uint4*>(dst) = __ldcg(reinterpret_cast<const uint4*>(src));
+    }
+    const int nt = (nk + 127) >> 7;
+    for (int i = nk * 16 + tid; i < nt * 128 * 16; i += kThreads) {  // (row, half, chunk) triples
+        const int row = i >> 4, half = (i >> 3) & 1, j = i & 7;
+        *reinterpret_cast<uint4*>(sV + (uint32_t)(row >> 7) * kTileBytes + half * kChunk + sw128_off(row & 127, j)) =
+            make_uint4(0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    const bool run = s_ok && nk > 0;  // CTA-uniform
+
+    // S^T = K Q^T, one 128-key tile at a time, into TMEM columns [16t, 16t + 16)
+    if (run && tid == 0) {
+        tc_fence_after();
+        constexpr uint32_t idesc = idesc_bf16_f32(128, 16);
+        for (int t = 0; t < nt; ++t) {
+            const uint32_t kt = smem_u32(sK + t * kTileBytes);
+            const uint32_t qt = smem_u32(sQ);
+#pragma unroll
+            for (int kk = 0; kk < kDH / 16; ++kk) {
+                const uint64_t ad = sw128_kmajor_desc(kt + (kk >> 2) * kChunk) + 2 * (kk & 3);
+                const uint64_t bd = sw128_kmajor_desc(qt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
+                umma_bf16_ss(tmem + t * 16, ad, bd, idesc, kk > 0 ? 1u : 0u);
+            }
+        }
+        umma_commit(&bar_mma);
+    }
+    float s[3][G];
+    float m_loc[G], l_loc[G];
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) m_loc[hh] = -INFINITY, l_loc[hh] = 0.f;
+    if (run) {
+        if (!mbar_wait(&bar_mma, 0)) s_ok = 0;
+        tc_fence_after();
+        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+        for (int t = 0; t < 3; ++t) {
+            if (t < nt) {
+                uint32_t r[16];
+                tmem_ld16(trow + t * 16, r);
+                const bool valid = t * 128 + warp * 32 + lane < nk;
+#pragma unroll
+                for (int hh = 0; hh < G; ++hh) {
+                    s[t][hh] = valid ? __uint_as_float(r[hh]) * p.scale_log2 : -INFINITY;
+                    m_loc[hh] = fmaxf(m_loc[hh], s[t][hh]);
+                }
+            } else {
+#pragma unroll
+                for (int hh = 0; hh < G; ++hh) s[t][hh] = -INFINITY;
+            }
+        }
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            float v = m_loc[hh];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+            if (lane == 0) red_m[warp][hh] = v;
+        }
+    }
+    __syncthreads();
+    if (run) {
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh)
+            m_loc[hh] = fmaxf(fmaxf(red_m[0][hh], red_m[1][hh]), fmaxf(red_m[2][hh], red_m[3][hh]));
+        // P^T[hh][key] = exp2(s - max) as bf16, swizzled K-major rows of 128 keys per tile
+        const int ki = warp * 32 + lane;  // key within the tile
+#pragma unroll
+        for (int t = 0; t < 3; ++t) {
+            if (t < nt) {
+                uint8_t* pt = sP + t * kPTileBytes + (ki >> 6) * (16 * 128);
+#pragma unroll
+                for (int hh = 0; hh < G; ++hh) {
+                    const float pe = s[t][hh] == -INFINITY ? 0.f : ex2_approx(s[t][hh] - m_loc[hh]);
+                    const bf16 pb = __float2bfloat16_rn(pe);
+                    l_loc[hh] += pe;
+                    *reinterpret_cast<bf16*>(pt + sw128_off(hh, (ki & 63) >> 3) + (ki & 7) * 2) = pb;
+                }
+            }
+        }
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            float v = l_loc[hh];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+            if (lane == 0) red_l[warp][hh] = v;
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+    }
+    __syncthreads();
+    // O^T = V^T P^T into TMEM columns [48, 64): A = V tile read MN-major (M = d_h), B = P^T
+    if (run && tid == 0) {
+        tc_fence_after();
+        constexpr uint32_t idesc = idesc_bf16_f32(128, 16) | (1u << 15);
+        for (int t = 0; t < nt; ++t) {
+            const uint32_t vt = smem_u32(sV + t * kTileBytes);
+            const uint32_t pt = smem_u32(sP + t * kPTileBytes);
+#pragma unroll
+            for (int kk = 0; kk < 128 / 16; ++kk) {
+                const uint64_t ad = sw128_mnmajor_desc(vt + kk * 16 * 128, kChunk);
+                const uint64_t bd = sw128_kmajor_desc(pt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
+                umma_bf16_ss(tmem + kOCol, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
+            }
+        }
+        umma_commit(&bar_mma);
+    }
+    if (run) {
+        if (!mbar_wait(&bar_mma, 1)) s_ok = 0;
+        tc_fence_after();
+        uint32_t r[16];
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + kOCol, r);
+        const int d = warp * 32 + lane;
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) c_o[hh * kDH + d] = __uint_as_float(r[hh]);
+        if (tid < G) {
+            c_m[tid] = m_loc[tid];
+            c_l[tid] = red_l[0][tid] + red_l[1][tid] + red_l[2][tid] + red_l[3][tid];
+        }
+    } else {
+        for (int i = tid; i < G * kDH; i += kThreads) c_o[i] = 0.f;
+        if (tid < G) {
+            c_m[tid] = -INFINITY;
+            c_l[tid] = 0.f;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+    if (!s_ok && tid == 0) set_status(p.status, kDevTimeout);
+    cluster_sync_all();  // every CTA's (c_m, c_l, c_o) is complete and visible to the cluster
+    const int per_cta = G * kDH / p.cs;
+    if (tid < per_cta) {
+        const int e = rank * per_cta + tid;
+        const int hh = e / kDH;
+        float mr[kMaxCs], lr[kMaxCs], orr[kMaxCs];
+#pragma unroll
+        for (int r = 0; r < kMaxCs; ++r) {
+            if (r < p.cs) {
+                mr[r] = ld_dsmem_f32(&c_m[hh], (uint32_t)r);
+                lr[r] = ld_dsmem_f32(&c_l[hh], (uint32_t)r);
+                orr[r] = ld_dsmem_f32(&c_o[e], (uint32_t)r);
+            }
+        }
+        float mx = -INFINITY;
+#pragma unroll
+        for (int r = 0; r < kMaxCs; ++r)
+            if (r < p.cs) mx = fmaxf(mx, mr[r]);
+        float lt = 0.f, ot = 0.f;
+#pragma unroll
+        for (int r = 0; r < kMaxCs; ++r) {
+            if (r < p.cs && mr[r] != -INFINITY) {
+                const float cw = ex2_approx(mr[r] - mx);
+                lt = fmaf(lr[r], cw, lt);
+                ot = fmaf(orr[r], cw, ot);
+            }
+        }
+        p.out[(size_t)kvh * G * kDH + e] = __float2bfloat16_rn(ot / lt);
+    }
+    cluster_sync_all();  // keep this CTA's shared memory alive until the cluster has read it
+}
+
+template <int G>
+cudaError_t prepare(int cs, size_t smem) {
+    cudaError_t e =
+        cudaFuncSetAttribute(attn_decode_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess && cs > 8)
+        e = cudaFuncSetAttribute(attn_decode_tc_kernel<G>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
+}
+
+template <int G>
+cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTcParams& p, cudaStream_t s, bool pdl) {
+    const size_t smem = smem_layout(p.nt).total;
+    static size_t attr_smem = 0;
+    static int attr_cs = 0;
+    if (smem > attr_smem || p.cs > attr_cs) {
+        cudaError_t e = prepare<G>(p.cs, smem);
+        if (e != cudaSuccess) return e;
+        attr_smem = smem > attr_smem ? smem : attr_smem;
+        attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.cs, p.Hkv);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = p.cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, attn_decode_tc_kernel<G>, tk, tv, p);
+}
+
+template <int G>
+bool plan(int Hkv, int max_ctx, int* cs, int* nt) {
+    for (int c : {16, 8}) {
+        const int keys = (max_ctx + c - 1) / c;
+        const int t = (keys + 127) / 128;
+        if (t > 3) continue;
+        const size_t smem = smem_layout(t).total;
+        if (prepare<G>(c, smem) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(c, Hkv);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = c;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, attn_decode_tc_kernel<G>, &cfg) != cudaSuccess) {
+            cudaGetLastError();
+            n = 0;
+        }
+        if (n >= 1) {
+            *cs = c;
+            *nt = t;
+            return true;
+        }
+    }
+    return false;
+}
+
+}  // namespace
+
+bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* nt) {
+    if (dh != kDH) return false;
+    switch (group) {
+        case 1: return plan<1>(Hkv, max_ctx, cs, nt);
+        case 2: return plan<2>(Hkv, max_ctx, cs, nt);
+        case 4: return plan<4>(Hkv, max_ctx, cs, nt);
+        case 8: return plan<8>(Hkv, max_ctx, cs, nt);
+    }
+    return false;
+}
+
+cudaError_t launch_attn_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, int group, const AttnDecTcParams& p,
+                                  cudaStream_t s, bool pdl) {
+    switch (group) {
+        case 1: return launch<1>(tk, tv, p, s, pdl);
+        case 2: return launch<2>(tk, tv, p, s, pdl);
+        case 4: return launch<4>(tk, tv, p, s, pdl);
+        case 8: return launch<8>(tk, tv, p, s, pdl);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace vla

@@ -104,16 +104,35 @@ struct DecodeDims {
 };
 struct DecodeWork {
     float* q;          // [H*dh] fp32 (post-RoPE query)
-    float* part_o;     // [splits][H][dh]
-    float* part_ml;    // [splits][H][2]
     bf16* attn;        // [H*dh]
     bf16* x_mid;       // [D]
     bf16* m;           // [F_pad]
     const float2* rope;
     unsigned* status;
-    unsigned* tickets;  // [Hkv] split-merge counters, zero between launches
-    int splits;
+    int attn_tc;                         // 1: tcgen05 kernel (attn_cap = tiles), 0: CUDA-core kernel
+    int attn_cs, attn_cap, attn_stages;  // from plan_decode_attention(_tc)
 };
+// Decode attention on tcgen05 (head_dim 128): one cluster of `cs` CTAs per KV head, each
+// holding up to nt tiles of 128 keys. K/V tensor maps: 3-D [Hkv][max_ctx][128] bf16 maps of the
+// layer's cache planes with 32-row boxes (make_tmap_bf16_3d).
+struct AttnDecTcParams {
+    const float* q;     // [H*dh] post-RoPE query, fp32
+    const bf16* kc;     // layer base [Hkv][max_ctx][dh] (the new token's row is read directly)
+    const bf16* vc;
+    const int* d_len;   // position of the new token; context = d_len + 1
+    int H, Hkv, max_ctx, cs, nt;
+    float scale_log2;
+    bf16* out;          // [H*dh]
+    unsigned* status;
+};
+bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* nt);
+cudaError_t launch_attn_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, int group, const AttnDecTcParams& p,
+                                  cudaStream_t s, bool pdl);
+
+// Decode-attention launch plan for contexts up to max_ctx: cluster size (CTAs per KV head),
+// keys per shared-memory stage and stage count.
+cudaError_t plan_decode_attention(int dh, int group, int Hkv, int max_ctx, int* cs, int* cap, int* stages);
+
 // Optional per-launch hook (measurement): called with (ctx, stage, begin) around each kernel.
 struct StageHook {
     void (*fn)(void* ctx, int stage, bool begin);
@@ -126,8 +145,11 @@ struct StageHook {
 // Stage ids of the decode kernels (match VLA_STAGE_DEC_* in vla_prefix.h)
 enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecO = 9, kStageDecGateUp = 10, kStageDecDown = 11 };
 
+// pdl_first: the layer's first kernel may overlap the previous kernel in the stream (set when
+// that kernel is the previous layer's down projection). The layer's later kernels always use
+// programmatic dependent launch unless a stage hook is installed.
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
-                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook);
+                                bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook, bool pdl_first);
 
 // d_len[i] += 1 for i < count (after all layers of a decode step have read their position)
 cudaError_t launch_advance_lengths(int* d_len, int count, cudaStream_t stream);

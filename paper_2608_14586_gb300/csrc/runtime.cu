@@ -115,11 +115,10 @@ struct vla_prefix {
     bf16 *ws_q = nullptr, *ws_attn = nullptr, *ws_xmid = nullptr, *ws_m = nullptr;
     float* ws_rinv = nullptr;
     // decode workspace
-    float *dq = nullptr, *d_part_o = nullptr, *d_part_ml = nullptr;
+    float* dq = nullptr;
     bf16 *d_attn = nullptr, *d_xmid = nullptr, *d_m = nullptr;
-    int dec_splits;
+    int attn_tc = 0, attn_cs = 0, attn_cap = 0, attn_stages = 0;  // decode-attention plan
     unsigned* d_status = nullptr;
-    unsigned* d_tickets = nullptr;
     int last_launches = 0;
     // measurement: event pairs around each kernel while timing is enabled
     unsigned timing = 0;  // bit s: time the kernels of stage s
@@ -173,13 +172,10 @@ void free_prefix(vla_prefix* p) {
     cudaFree(p->ws_m);
     cudaFree(p->ws_rinv);
     cudaFree(p->dq);
-    cudaFree(p->d_part_o);
-    cudaFree(p->d_part_ml);
     cudaFree(p->d_attn);
     cudaFree(p->d_xmid);
     cudaFree(p->d_m);
     cudaFree(p->d_status);
-    cudaFree(p->d_tickets);
     for (cudaEvent_t e : p->ev_pool) cudaEventDestroy(e);
     for (auto& g : p->graphs) cudaGraphExecDestroy(g.exec);
     if (p->cap_stream) cudaStreamDestroy(p->cap_stream);
@@ -296,17 +292,12 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
                  n_d = (size_t)D * p->F_pad;
     const size_t per_layer = n_qkv + n_o + n_gu + n_d;
     const int T = cfg->max_ctx;
-    // decode attention: two CTAs per SM over the KV heads, and few enough keys per split for
-    // its K and V rows to sit in 160 KB of shared memory
-    const int keys_in_smem = 160 * 1024 / (4 * dh);
-    p->dec_splits = std::max((2 * p->num_sms + Hkv - 1) / Hkv, (T + keys_in_smem - 1) / keys_in_smem);
     bool ok = dmalloc(&p->weight_pool, per_layer * layer_count) && dmalloc(&p->rope, (size_t)T * dh / 2) &&
               dmalloc(&p->ws_q, (size_t)T * p->qc) && dmalloc(&p->ws_attn, (size_t)T * p->qc) &&
               dmalloc(&p->ws_xmid, (size_t)T * D) && dmalloc(&p->ws_m, (size_t)T * p->F_pad) &&
               dmalloc(&p->ws_rinv, (size_t)T) && dmalloc(&p->dq, (size_t)p->qc) &&
-              dmalloc(&p->d_part_o, (size_t)p->dec_splits * H * dh) &&
-              dmalloc(&p->d_part_ml, (size_t)p->dec_splits * H * 2) && dmalloc(&p->d_attn, (size_t)p->qc) &&
-              dmalloc(&p->d_xmid, (size_t)D) && dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1) && dmalloc(&p->d_tickets, (size_t)Hkv) &&
+              dmalloc(&p->d_attn, (size_t)p->qc) && dmalloc(&p->d_xmid, (size_t)D) &&
+              dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1) &&
               dmalloc(&p->d_xin, (size_t)D) && dmalloc(&p->d_xout, (size_t)D);
     if (!ok) {
         cudaGetLastError();
@@ -314,7 +305,11 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         return VLA_ERR_OOM;
     }
     cudaError_t e = cudaMemset(p->d_status, 0, sizeof(unsigned));
-    if (e == cudaSuccess) e = cudaMemset(p->d_tickets, 0, sizeof(unsigned) * Hkv);
+    if (e == cudaSuccess) {
+        p->attn_tc = vla::plan_decode_attention_tc(dh, H / Hkv, Hkv, T, &p->attn_cs, &p->attn_cap) ? 1 : 0;
+        if (!p->attn_tc)
+            e = vla::plan_decode_attention(dh, H / Hkv, Hkv, T, &p->attn_cs, &p->attn_cap, &p->attn_stages);
+    }
     if (e == cudaSuccess) e = vla::launch_rope_table(p->rope, T, dh, (double)cfg->rope_base, 0);
     p->layers.resize(layer_count);
     for (int l = 0; l < layer_count && e == cudaSuccess; ++l) {
@@ -576,8 +571,8 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
     }
     vla::DecodeDims dims = {D, p->cfg.n_heads, p->cfg.n_kv_heads, p->cfg.head_dim, p->F_pad, kv->max_ctx,
                             p->cfg.rms_eps};
-    vla::DecodeWork w = {p->dq,      p->d_part_o, p->d_part_ml, p->d_attn,      p->d_xmid,
-                         p->d_m,     p->rope,     p->d_status,  p->d_tickets, p->dec_splits};
+    vla::DecodeWork w = {p->dq,      p->d_attn,  p->d_xmid,  p->d_m,      p->rope,
+                         p->d_status, p->attn_tc, p->attn_cs, p->attn_cap, p->attn_stages};
     const int nl = layer_end - layer_begin;
     // enqueue the whole step on stream s, reading x_in and chaining through x_out
     auto enqueue = [&](const bf16* x_in, bf16* x_out, cudaStream_t s, const vla::StageHook& hook) {
@@ -586,7 +581,8 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
             const LayerDev& ld = p->layers[l];
             vla::DecodeLayer L = {ld.w_qkv, ld.w_o, ld.w_gu, ld.w_d, kv->k_plane(l), kv->v_plane(l),
                                   kv->d_len + (l - kv->lb)};
-            e = vla::launch_decode_layer(L, dims, w, l == layer_begin ? x_in : x_out, x_out, p->num_sms, s, hook);
+            e = vla::launch_decode_layer(L, dims, w, l == layer_begin ? x_in : x_out, x_out, p->num_sms, s, hook,
+                                         l > layer_begin);
         }
         if (e == cudaSuccess) e = vla::launch_advance_lengths(kv->d_len + (layer_begin - kv->lb), nl, s);
         return e;
