@@ -645,7 +645,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
         t.Hkv = d.Hkv;
         t.max_ctx = d.max_ctx;
         t.cs = w.attn_cs;
-        t.nt = w.attn_cap;
+        t.rows = w.attn_cap;
         t.scale_log2 = a.scale_log2;
         t.out = w.attn;
         t.status = w.status;

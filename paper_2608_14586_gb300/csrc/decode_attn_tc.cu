@@ -3,7 +3,8 @@
 // One thread-block cluster of `cs` CTAs per KV head g; CTA rank r owns the contiguous key range
 // [r*ceil(ctx/cs), ...) of the context (Sec. 3.2's causal attention at one query position,
 // split over keys). Per CTA, for the G query heads of the GQA group:
-//   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory.
+//   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory
+//      sized to the range (two CTAs fit on an SM, so all Hkv clusters of 16 are co-resident).
 //      Rows that predate this step are requested before griddepcontrol.wait, so the copy
 //      overlaps the QKV kernel; the new token's row is written over its slot afterwards.
 //   2. S^T = K Q^T on tcgen05 (M = 128 keys per tile, N = 16 >= G heads, K = d_h), fp32 in TMEM.
@@ -26,6 +27,7 @@ constexpr int kThreads = 128;
 constexpr int kBoxRows = 32;
 constexpr uint32_t kChunk = 128u * 128u;            // [128 rows][64 bf16] per d_h half
 constexpr uint32_t kTileBytes = 2u * kChunk;        // 128 keys x 128 d_h
+constexpr int kMaxRows = 384;                       // keys per CTA (3 tiles)
 constexpr uint32_t kQBytes = 2u * 16u * 128u;       // [16 rows][128] as two halves of 64
 constexpr uint32_t kPTileBytes = 2u * 16u * 128u;   // [16 heads][128 keys] as two halves of 64
 constexpr uint32_t kBoxBytes = kBoxRows * 128u;     // one [32 rows][64] box
@@ -47,18 +49,29 @@ VLA_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 // byte offset of (row, 16-byte chunk j) inside a 128-byte-swizzled tile of 128-byte rows
 VLA_DEV uint32_t sw128_off(int row, int j) { return (uint32_t)row * 128u + ((uint32_t)(j ^ (row & 7)) << 4); }
 
+// Shared memory for `rows` keys per CTA (a multiple of 32): K and V as tiles of 128 keys, the
+// last tile holding only the remaining rows; tile t's two d_h halves are rows_t * 128 bytes
+// apart. The S MMA of a partial tile reads all 128 rows of each half window, past the tile's
+// own rows into the buffers that follow (never past the allocation, since rows_t >= 32);
+// those keys are masked, and the O MMA reads only the 16-key steps that hold keys.
 struct Smem {
     uint32_t off_k, off_v, off_q, off_p, total;
 };
 
-__host__ __device__ inline Smem smem_layout(int nt) {
+__host__ __device__ inline Smem smem_layout(int rows) {
     Smem s;
     s.off_k = 0;
-    s.off_v = nt * kTileBytes;
-    s.off_q = 2 * nt * kTileBytes;
+    s.off_v = (uint32_t)rows * 256u;
+    s.off_q = 2u * s.off_v;
     s.off_p = s.off_q + kQBytes;
-    s.total = s.off_p + nt * kPTileBytes + 1024;  // + alignment slack
+    s.total = s.off_p + (uint32_t)((rows + 127) / 128) * kPTileBytes + 1024;  // + alignment slack
     return s;
+}
+
+// byte offset of d_h half `half` of tile t for `rows` allocated keys
+__host__ __device__ inline uint32_t half_off(int rows, int t, int half) {
+    const int rt = min(128, rows - 128 * t);
+    return (uint32_t)t * kTileBytes + (uint32_t)half * (uint32_t)rt * 128u;
 }
 
 template <int G>
@@ -74,7 +87,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ int s_ok;
     const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
     uint8_t* smem = smem_raw + pad;
-    const Smem L = smem_layout(p.nt);
+    const Smem L = smem_layout(p.rows);
     uint8_t* sK = smem + L.off_k;
     uint8_t* sV = smem + L.off_v;
     uint8_t* sQ = smem + L.off_q;
@@ -86,7 +99,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ctx = *p.d_len + 1;
     const int per = (ctx + p.cs - 1) / p.cs;
     const int kb = rank * per;
-    const int nk = max(0, min(min(ctx, kb + per) - kb, p.nt * 128));
+    const int nk = max(0, min(min(ctx, kb + per) - kb, p.rows));
     const int nbox = (nk + kBoxRows - 1) / kBoxRows;
     const int new_row = ctx - 1 - kb;  // slot of the token written by the QKV kernel
 
@@ -103,7 +116,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_relinquish();
     }
     // zero Q rows >= G and the P^T tiles (rows >= G stay zero; rows < G are rewritten)
-    for (uint32_t i = tid; i < (kQBytes + p.nt * kPTileBytes) / 16; i += kThreads)
+    for (uint32_t i = tid; i < (L.total - 1024 - L.off_q) / 16; i += kThreads)
         reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0u, 0u, 0u, 0u);
     tc_fence_before();
     __syncthreads();
@@ -112,11 +125,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tid == 0) {
         mbar_arrive_expect_tx(&bar_kv, (uint32_t)nbox * 4u * kBoxBytes);
         for (int b = 0; b < nbox; ++b) {
-            const uint32_t dst = (uint32_t)(b >> 2) * kTileBytes + (uint32_t)(b & 3) * kBoxBytes;
             const int y = kb + b * kBoxRows;
             for (int c = 0; c < 2; ++c) {
-                tma_load_3d(sK + dst + c * kChunk, &tmK, &bar_kv, c * 64, y, kvh);
-                tma_load_3d(sV + dst + c * kChunk, &tmV, &bar_kv, c * 64, y, kvh);
+                const uint32_t dst = half_off(p.rows, b >> 2, c) + (uint32_t)(b & 3) * kBoxBytes;
+                tma_load_3d(sK + dst, &tmK, &bar_kv, c * 64, y, kvh);
+                tma_load_3d(sV + dst, &tmV, &bar_kv, c * 64, y, kvh);
             }
         }
     }
@@ -137,14 +150,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (new_row >= 0 && new_row < nk && tid < 32) {
         const int half = tid >> 4, j = (tid >> 1) & 7, which = tid & 1;  // 2 halves x 8 chunks x {K, V}
         const bf16* src = (which ? p.vc : p.kc) + ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + half * 64 + j * 8;
-        uint8_t* dst = (which ? sV : sK) + (uint32_t)(new_row >> 7) * kTileBytes + half * kChunk +
-                       sw128_off(new_row & 127, j);
+        uint8_t* dst = (which ? sV : sK) + half_off(p.rows, new_row >> 7, half) + sw128_off(new_row & 127, j);
         *reinterpret_cast<uint4*>(dst) = __ldcg(reinterpret_cast<const uint4*>(src));
     }
     const int nt = (nk + 127) >> 7;
-    for (int i = nk * 16 + tid; i < nt * 128 * 16; i += kThreads) {  // (row, half, chunk) triples
+    const int zero_end = min(p.rows, (nk + 31) & ~31);  // rows the O MMA may read
+    for (int i = nk * 16 + tid; i < zero_end * 16; i += kThreads) {  // (row, half, chunk) triples
         const int row = i >> 4, half = (i >> 3) & 1, j = i & 7;
-        *reinterpret_cast<uint4*>(sV + (uint32_t)(row >> 7) * kTileBytes + half * kChunk + sw128_off(row & 127, j)) =
+        *reinterpret_cast<uint4*>(sV + half_off(p.rows, row >> 7, half) + sw128_off(row & 127, j)) =
             make_uint4(0u, 0u, 0u, 0u);
     }
     fence_proxy_async_smem();
@@ -156,11 +169,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         constexpr uint32_t idesc = idesc_bf16_f32(128, 16);
         for (int t = 0; t < nt; ++t) {
-            const uint32_t kt = smem_u32(sK + t * kTileBytes);
             const uint32_t qt = smem_u32(sQ);
 #pragma unroll
             for (int kk = 0; kk < kDH / 16; ++kk) {
-                const uint64_t ad = sw128_kmajor_desc(kt + (kk >> 2) * kChunk) + 2 * (kk & 3);
+                const uint64_t ad = sw128_kmajor_desc(smem_u32(sK + half_off(p.rows, t, kk >> 2))) + 2 * (kk & 3);
                 const uint64_t bd = sw128_kmajor_desc(qt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
                 umma_bf16_ss(tmem + t * 16, ad, bd, idesc, kk > 0 ? 1u : 0u);
             }
@@ -235,11 +247,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         constexpr uint32_t idesc = idesc_bf16_f32(128, 16) | (1u << 15);
         for (int t = 0; t < nt; ++t) {
-            const uint32_t vt = smem_u32(sV + t * kTileBytes);
+            const uint32_t vt = smem_u32(sV + half_off(p.rows, t, 0));
+            const uint32_t vstride = half_off(p.rows, t, 1) - half_off(p.rows, t, 0);
             const uint32_t pt = smem_u32(sP + t * kPTileBytes);
-#pragma unroll
-            for (int kk = 0; kk < 128 / 16; ++kk) {
-                const uint64_t ad = sw128_mnmajor_desc(vt + kk * 16 * 128, kChunk);
+            const int steps = (min(128, nk - 128 * t) + 15) >> 4;  // 16-key steps holding keys
+            for (int kk = 0; kk < steps; ++kk) {
+                const uint64_t ad = sw128_mnmajor_desc(vt + kk * 16 * 128, vstride);
                 const uint64_t bd = sw128_kmajor_desc(pt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
                 umma_bf16_ss(tmem + kOCol, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
             }
@@ -315,7 +328,7 @@ cudaError_t prepare(int cs, size_t smem) {
 
 template <int G>
 cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTcParams& p, cudaStream_t s, bool pdl) {
-    const size_t smem = smem_layout(p.nt).total;
+    const size_t smem = smem_layout(p.rows).total;
     static size_t attr_smem = 0;
     static int attr_cs = 0;
     if (smem > attr_smem || p.cs > attr_cs) {
@@ -341,13 +354,16 @@ cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTc
     return cudaLaunchKernelEx(&cfg, attn_decode_tc_kernel<G>, tk, tv, p);
 }
 
+// Cluster size 16 (else 8) with each CTA holding ceil(max_ctx / cs) keys; preferred when all
+// Hkv clusters can be resident at once, which needs two CTAs per SM (so the keys of a CTA are
+// allocated to the next 32, not to whole tiles).
 template <int G>
-bool plan(int Hkv, int max_ctx, int* cs, int* nt) {
+bool plan(int Hkv, int max_ctx, int* cs, int* rows) {
+    int best_c = 0, best_rows = 0, best_n = 0;
     for (int c : {16, 8}) {
-        const int keys = (max_ctx + c - 1) / c;
-        const int t = (keys + 127) / 128;
-        if (t > 3) continue;
-        const size_t smem = smem_layout(t).total;
+        const int r = ((max_ctx + c - 1) / c + 31) & ~31;
+        if (r > kMaxRows) continue;
+        const size_t smem = smem_layout(r).total;
         if (prepare<G>(c, smem) != cudaSuccess) {
             cudaGetLastError();
             continue;
@@ -368,24 +384,28 @@ bool plan(int Hkv, int max_ctx, int* cs, int* nt) {
             cudaGetLastError();
             n = 0;
         }
-        if (n >= 1) {
+        if (n >= Hkv) {
             *cs = c;
-            *nt = t;
+            *rows = r;
             return true;
         }
+        if (n > best_n) best_c = c, best_rows = r, best_n = n;
     }
-    return false;
+    if (best_n == 0) return false;
+    *cs = best_c;
+    *rows = best_rows;
+    return true;
 }
 
 }  // namespace
 
-bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* nt) {
+bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* rows) {
     if (dh != kDH) return false;
     switch (group) {
-        case 1: return plan<1>(Hkv, max_ctx, cs, nt);
-        case 2: return plan<2>(Hkv, max_ctx, cs, nt);
-        case 4: return plan<4>(Hkv, max_ctx, cs, nt);
-        case 8: return plan<8>(Hkv, max_ctx, cs, nt);
+        case 1: return plan<1>(Hkv, max_ctx, cs, rows);
+        case 2: return plan<2>(Hkv, max_ctx, cs, rows);
+        case 4: return plan<4>(Hkv, max_ctx, cs, rows);
+        case 8: return plan<8>(Hkv, max_ctx, cs, rows);
     }
     return false;
 }

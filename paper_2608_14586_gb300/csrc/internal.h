@@ -109,23 +109,23 @@ struct DecodeWork {
     bf16* m;           // [F_pad]
     const float2* rope;
     unsigned* status;
-    int attn_tc;                         // 1: tcgen05 kernel (attn_cap = tiles), 0: CUDA-core kernel
+    int attn_tc;                         // 1: tcgen05 kernel (attn_cap = keys per CTA), 0: CUDA-core kernel
     int attn_cs, attn_cap, attn_stages;  // from plan_decode_attention(_tc)
 };
 // Decode attention on tcgen05 (head_dim 128): one cluster of `cs` CTAs per KV head, each
-// holding up to nt tiles of 128 keys. K/V tensor maps: 3-D [Hkv][max_ctx][128] bf16 maps of the
+// holding up to `rows` keys (a multiple of 32, at most 384). K/V tensor maps: 3-D [Hkv][max_ctx][128] bf16 maps of the
 // layer's cache planes with 32-row boxes (make_tmap_bf16_3d).
 struct AttnDecTcParams {
     const float* q;     // [H*dh] post-RoPE query, fp32
     const bf16* kc;     // layer base [Hkv][max_ctx][dh] (the new token's row is read directly)
     const bf16* vc;
     const int* d_len;   // position of the new token; context = d_len + 1
-    int H, Hkv, max_ctx, cs, nt;
+    int H, Hkv, max_ctx, cs, rows;
     float scale_log2;
     bf16* out;          // [H*dh]
     unsigned* status;
 };
-bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* nt);
+bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* rows);
 cudaError_t launch_attn_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, int group, const AttnDecTcParams& p,
                                   cudaStream_t s, bool pdl);
 
