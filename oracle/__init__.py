@@ -24,6 +24,7 @@ from .decoder import (  # noqa: F401
     apply_rope,
     attention_weights,
     block_forward,
+    block_forward_rows,
     boundary_bytes,
     boundary_transfer,
     bf16_to_f64,

@@ -212,6 +212,36 @@ def block_forward(x: np.ndarray, w: LayerWeights, cache: KVCache, layer: int, sh
     return y
 
 
+def block_forward_rows(x: np.ndarray, w: LayerWeights, shape, rows, p0: int = 0,
+                       ctx_k: np.ndarray | None = None, ctx_v: np.ndarray | None = None):
+    """Block B_l on x [M, D] at positions p0.., evaluated only at the query rows ``rows``.
+
+    Same stages as block_forward: every row's key and value are formed (attention needs
+    them), but the query, attention output, projections and feed-forward are computed only
+    for the selected rows. ``ctx_k`` / ``ctx_v`` [H_kv, p0, d_h] hold the cached positions
+    before p0 (post-rotary keys). Returns (y [len(rows), D], k [H_kv, M, d_h], v [H_kv, M, d_h])
+    where k, v are this call's cache entries.
+    """
+    M, D = x.shape
+    H, Hkv, dh = shape.n_heads, shape.n_kv_heads, shape.head_dim
+    rows = np.asarray(rows, dtype=np.int64)
+    pos = p0 + np.arange(M)
+    u = rms_norm(x, w.g_attn, shape.rms_eps)
+    k = apply_rope((u @ w.w_k.T).reshape(M, Hkv, dh), pos, shape.rope_base).transpose(1, 0, 2)
+    v = (u @ w.w_v.T).reshape(M, Hkv, dh).transpose(1, 0, 2)
+    if p0 > 0:
+        k_all = np.concatenate([ctx_k[:, :p0], k], axis=1)
+        v_all = np.concatenate([ctx_v[:, :p0], v], axis=1)
+    else:
+        k_all, v_all = k, v
+    q = apply_rope((u[rows] @ w.w_q.T).reshape(len(rows), H, dh), pos[rows], shape.rope_base)
+    o = causal_gqa_attention(q, k_all, v_all, pos[rows], Hkv)
+    xm = x[rows] + o.reshape(len(rows), H * dh) @ w.w_o.T
+    u2 = rms_norm(xm, w.g_mlp, shape.rms_eps)
+    y = xm + swiglu(u2 @ w.w_gate.T, u2 @ w.w_up.T) @ w.w_down.T
+    return y, k, v
+
+
 def prefix_forward(x: np.ndarray, weights, layer_begin: int, layer_end: int, cache: KVCache,
                    shape, per_block: list | None = None) -> np.ndarray:
     """Blocks [layer_begin, layer_end) applied in order (Eq. 5 for layer_begin = 0).

@@ -1,0 +1,149 @@
+"""The boundary hand-off of Eq. 6 / Eq. 11 on the GPU: the GPU range [0, k) writes h^(k), a
+side stream copies it into page-locked host memory while the main stream continues, and
+the split point may change from frame to frame (same KV cache, no reallocation). Also the
+argument checks of the C ABI against a live prefix object."""
+import ctypes
+
+import numpy as np
+import pytest
+
+import synth
+from helpers import sync, Model, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _bits(t):
+    import torch
+    return t.detach().contiguous().view(torch.int16).cpu().numpy()
+
+
+def test_frames_with_overlapped_boundary_copies_and_per_frame_split(vla_lib):
+    """Four 3072-token frames (6 x 448 visual + 384 text rows) through an 8-block 7B-class
+    stack, double-buffered: frame f's boundary copy overlaps frame f's suffix range and
+    frame f+1's prefix. Each frame uses its own split point; the host copy of h^(k) and the
+    range output equal single-stream reference runs bit for bit."""
+    import torch
+    vla = vla_lib
+    s, L, M = synth.B7, 8, 3072
+    ks = [2, 4, 6, 4]
+    m = Model(s, L, 0, M)
+    try:
+        main = torch.cuda.current_stream()
+        side = torch.cuda.Stream()
+        kvs = [vla.vla_kv_create(m.handle, 0, L, M) for _ in range(2)]
+        hdev = [torch.empty((M, s.hidden), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+        ydev = [torch.empty_like(hdev[0]) for _ in range(2)]
+        pinned = [torch.empty((M, s.hidden), dtype=torch.bfloat16, pin_memory=True) for _ in range(2)]
+        ready = [torch.cuda.Event() for _ in range(2)]
+        done = [torch.cuda.Event() for _ in range(2)]
+        for e in done:
+            e.record(side)  # creates the event handle the library records into
+        xs = [to_dev(synth.hidden_states(M, s.hidden, f, 2688, 1.0)) for f in range(4)]
+        # references: one stream, fresh caches, no overlap
+        kv_ref = vla.vla_kv_create(m.handle, 0, L, M)
+        h_ref, y_ref = [], []
+        for f in range(4):
+            h = torch.empty_like(hdev[0])
+            y = torch.empty_like(hdev[0])
+            vla.vla_kv_reset(kv_ref)
+            vla.vla_prefix_prefill(m.handle, xs[f], M, 0, ks[f], kv_ref, h)
+            vla.vla_kv_reset(kv_ref)
+            vla.vla_prefix_prefill(m.handle, xs[f], M, 0, L, kv_ref, y)
+            h_ref.append(h)
+            y_ref.append(y)
+        sync(120)
+        ref_h = [_bits(h) for h in h_ref]
+        ref_y = [_bits(y) for y in y_ref]
+
+        def check(f):
+            b = f % 2
+            done[b].synchronize()
+            np.testing.assert_array_equal(pinned[b].view(torch.int16).numpy(), ref_h[f])
+
+        for f in range(4):
+            b = f % 2
+            if f >= 2:
+                check(f - 2)  # buffer b's previous copy has landed and is verified before reuse
+            vla.vla_kv_reset(kvs[b], main)
+            vla.vla_prefix_prefill(m.handle, xs[f], M, 0, ks[f], kvs[b], hdev[b], main)
+            ready[b].record(main)
+            vla.vla_boundary_to_host(hdev[b], M, s.hidden, pinned[b], side, ready[b], done[b])
+            vla.vla_prefix_prefill(m.handle, hdev[b], M, ks[f], L, kvs[b], ydev[b], main)
+            main.wait_event(done[b])  # hdev[b] is rewritten two frames later
+            if f >= 2:
+                sync(120)
+                np.testing.assert_array_equal(_bits(ydev[b]), ref_y[f])
+        check(2)
+        check(3)
+        sync(120)
+        np.testing.assert_array_equal(_bits(ydev[1]), ref_y[3])
+        assert vla.vla_last_async_error(m.handle) == 0
+        for kv in kvs + [kv_ref]:
+            vla.vla_kv_destroy(kv)
+    finally:
+        m.close()
+
+
+def test_abi_errors_on_a_live_prefix(vla_lib):
+    import torch
+    vla = vla_lib
+    s = synth.TINY
+    L, max_ctx = 3, 32
+    m = Model(s, L, 2, max_ctx)
+    other = Model(s, 1, 3, max_ctx)
+    try:
+        x = to_dev(synth.hidden_states(16, s.hidden, 2))
+        y = torch.empty_like(x)
+        kv = vla.vla_kv_create(m.handle, 0, 2, max_ctx)  # covers layers [0, 2) only
+
+        def status(fn, *a):
+            with pytest.raises(vla.VlaError) as ei:
+                fn(*a)
+            return ei.value.name
+
+        assert status(vla.vla_prefix_prefill, m.handle, x, 16, 0, 3, kv, y) == "VLA_ERR_RANGE"  # beyond the cache
+        assert status(vla.vla_prefix_prefill, m.handle, x, 16, 2, 1, kv, y) == "VLA_ERR_RANGE"  # reversed
+        assert status(vla.vla_prefix_prefill, m.handle, x, 16, 0, 4, kv, y) == "VLA_ERR_RANGE"  # beyond the model
+        assert status(vla.vla_kv_create, m.handle, 0, 4, max_ctx) in ("VLA_ERR_RANGE", "VLA_ERR_INVALID_ARG")
+        kv_other = vla.vla_kv_create(other.handle, 0, 1, max_ctx)
+        assert status(vla.vla_prefix_prefill, m.handle, x, 16, 0, 1, kv_other, y) == "VLA_ERR_INVALID_ARG"
+        # layer 0 advanced alone: a range starting at different lengths is refused
+        vla.vla_prefix_prefill(m.handle, x, 16, 0, 1, kv, y)
+        assert status(vla.vla_prefix_prefill, m.handle, x, 16, 0, 2, kv, y) == "VLA_ERR_RANGE"
+        vla.vla_prefix_prefill(m.handle, y, 16, 1, 2, kv, y)  # in place; layer 1 catches up
+        assert vla.vla_kv_length(kv) == 16
+        # 16 + 17 > 32 positions
+        x17 = to_dev(synth.hidden_states(17, s.hidden, 2))
+        assert status(vla.vla_prefix_prefill, m.handle, x17, 17, 0, 2, kv, torch.empty_like(x17)) == "VLA_ERR_KV_FULL"
+        # decode fills the cache to the last position, then refuses
+        one = torch.empty((1, s.hidden), dtype=torch.bfloat16, device="cuda")
+        for t in range(16):
+            vla.vla_prefix_decode(m.handle, to_dev(synth.decode_hidden(t, s.hidden, 2)), 0, 2, kv, one)
+        assert vla.vla_kv_length(kv) == 32
+        assert status(vla.vla_prefix_decode, m.handle, one, 0, 2, kv, one) == "VLA_ERR_KV_FULL"
+        # unaligned device pointers
+        raw = torch.empty(16 * s.hidden + 8, dtype=torch.bfloat16, device="cuda")
+        assert status(vla.vla_prefix_prefill, m.handle, raw.data_ptr() + 2, 16, 0, 2, kv, y) == "VLA_ERR_INVALID_ARG"
+        # pageable host memory is refused for the boundary copy; pinned memory is accepted
+        pageable = np.zeros((16, s.hidden), dtype=np.uint16)
+        assert status(vla.vla_boundary_to_host, y, 16, s.hidden, pageable.ctypes.data) == "VLA_ERR_NOT_PINNED"
+        pin = torch.empty((16, s.hidden), dtype=torch.bfloat16, pin_memory=True)
+        vla.vla_boundary_to_host(y, 16, s.hidden, pin)
+        sync()
+        np.testing.assert_array_equal(pin.view(torch.int16).numpy(), _bits(y))
+        # an empty range is a copy, needs no cache, and leaves lengths alone
+        z = torch.empty_like(x)
+        vla.vla_prefix_prefill(m.handle, x, 16, 2, 2, None, z)
+        sync()
+        assert torch.equal(z.view(torch.int16), x.view(torch.int16))
+        vla.vla_kv_reset(kv)
+        sync()
+        assert vla.vla_kv_length(kv) == 0
+        assert vla.vla_last_async_error(m.handle) == 0
+        assert ctypes.c_int(vla.vla_kv_layer_length(kv, 5)).value == -1
+        vla.vla_kv_destroy(kv)
+        vla.vla_kv_destroy(kv_other)
+    finally:
+        m.close()
+        other.close()

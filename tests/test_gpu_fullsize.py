@@ -1,0 +1,147 @@
+"""Full-size parity at the benchmark's shapes: the 16-block 7B-class prefix over a 2304-token
+frame (prefill) and 16-block decode against a 2304-position context.
+
+The float64 oracle cannot run the whole 16-block frame in seconds, so each block is checked
+teacher-forced: the oracle receives the block's GPU input (exact bf16 values) and evaluates
+the block at sampled query rows (all rows' keys and values, which attention needs, are
+formed in full). The chained GPU result is tied to the per-block calls by the partition
+identity of Eq. 6, checked bit for bit.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from helpers import sync, COS_FINAL, REL_L2_BLOCK, Model, cos_sim, from_dev, kv_planes, rel_l2, to_dev
+
+pytestmark = pytest.mark.gpu
+
+# query rows checked per block: both ends, the visual/text seam and a seeded spread
+_ROWS = sorted(set([0, 1, 319, 320, 1919, 1920, 2302, 2303] +
+                   np.random.default_rng(5).choice(2304, 24, replace=False).tolist()))
+
+
+def test_prefill_16_blocks_2304_tokens_teacher_forced_and_partition_identity(vla_lib):
+    import torch
+    vla = vla_lib
+    wl = synth.WORKLOADS["7b_prefix16_2304tok"]
+    s, L, M = wl.shape, wl.prefix_layers, wl.n_tokens
+    m = Model(s, L, wl.seed, M)
+    try:
+        xb = synth.hidden_states(M, s.hidden, wl.seed, wl.visual_tokens, wl.visual_scale)
+        # block by block: h[l] is block l's input
+        kv = vla.vla_kv_create(m.handle, 0, L, M)
+        h = [to_dev(xb)] + [torch.empty((M, s.hidden), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+        for l in range(L):
+            vla.vla_prefix_prefill(m.handle, h[l], M, l, l + 1, kv, h[l + 1])
+        # one call over [0, L) and a split at k = 8 (Eq. 6): identical bits
+        kv_full = vla.vla_kv_create(m.handle, 0, L, M)
+        y_full = torch.empty_like(h[0])
+        vla.vla_prefix_prefill(m.handle, h[0], M, 0, L, kv_full, y_full)
+        kv_split = vla.vla_kv_create(m.handle, 0, L, M)
+        hk = torch.empty_like(h[0])
+        y_split = torch.empty_like(h[0])
+        vla.vla_prefix_prefill(m.handle, h[0], M, 0, 8, kv_split, hk)
+        vla.vla_prefix_prefill(m.handle, hk, M, 8, L, kv_split, y_split)
+        sync(120)
+        assert vla.vla_last_async_error(m.handle) == 0
+        assert torch.equal(y_full.view(torch.int16), h[L].view(torch.int16))
+        assert torch.equal(y_split.view(torch.int16), h[L].view(torch.int16))
+        assert torch.equal(hk.view(torch.int16), h[8].view(torch.int16))
+        assert vla.vla_kv_length(kv) == M and vla.vla_kv_length(kv_full) == M
+        for l in range(L):
+            x_in = from_dev(h[l])
+            y_ref, k_ref, v_ref = oracle.block_forward_rows(x_in, m.w64(l), s, _ROWS)
+            got = from_dev(h[l + 1])[_ROWS]
+            assert rel_l2(got, y_ref) < REL_L2_BLOCK, l
+            assert cos_sim(got, y_ref) > COS_FINAL, l
+            K, V = kv_planes(vla, kv, l, s, M)
+            assert rel_l2(from_dev(K), k_ref) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(V), v_ref) < REL_L2_BLOCK, l
+            m.drop_w64()
+        for k in (kv, kv_full, kv_split):
+            vla.vla_kv_destroy(k)
+    finally:
+        m.close()
+
+
+def test_decode_16_blocks_context_2304_teacher_forced(vla_lib):
+    """Decode steps on the whole range (one captured graph) equal block-by-block decode bit
+    for bit; each block matches the oracle's decode step given the same input."""
+    import torch
+    vla = vla_lib
+    wl = synth.WORKLOADS["7b_decode16_ctx2304"]
+    s, L, ctx0 = wl.shape, wl.prefix_layers, wl.prefill_ctx
+    steps, max_ctx = 3, ctx0 + 64
+    m = Model(s, L, wl.seed, max_ctx)
+    try:
+        kv_a = vla.vla_kv_create(m.handle, 0, L, max_ctx)
+        kv_b = vla.vla_kv_create(m.handle, 0, L, max_ctx)
+        ctx_bits = [synth.random_kv(ctx0, s, wl.seed, l) for l in range(L)]
+        for kv in (kv_a, kv_b):
+            for l in range(L):
+                kt, vt = kv_planes(vla, kv, l, s, max_ctx)
+                kt[:, :ctx0].copy_(to_dev(ctx_bits[l][0]))
+                vt[:, :ctx0].copy_(to_dev(ctx_bits[l][1]))
+            sync()
+            vla.vla_kv_set_length(kv, ctx0)
+        out = torch.empty((1, s.hidden), dtype=torch.bfloat16, device="cuda")
+        hs = []  # hs[t][l]: block l's input at step t (GPU, block-by-block run)
+        for t in range(steps):
+            x = to_dev(synth.decode_hidden(t, s.hidden, wl.seed))
+            vla.vla_prefix_decode(m.handle, x, 0, L, kv_a, out)
+            h = [x] + [torch.empty_like(x) for _ in range(L)]
+            for l in range(L):
+                vla.vla_prefix_decode(m.handle, h[l], l, l + 1, kv_b, h[l + 1])
+            sync()
+            assert torch.equal(out.view(torch.int16), h[L].view(torch.int16)), t
+            hs.append([from_dev(v) for v in h])
+        assert vla.vla_last_async_error(m.handle) == 0
+        assert vla.vla_kv_length(kv_a) == ctx0 + steps and vla.vla_kv_length(kv_b) == ctx0 + steps
+        cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, max_ctx)
+        for l in range(L):
+            cache.fill(l, oracle.bf16_to_f64(ctx_bits[l][0]), oracle.bf16_to_f64(ctx_bits[l][1]))
+            for t in range(steps):
+                ref = oracle.block_forward(hs[t][l], m.w64(l), cache, l, s)
+                assert rel_l2(hs[t][l + 1], ref) < REL_L2_BLOCK, (l, t)
+            m.drop_w64()
+        vla.vla_kv_destroy(kv_a)
+        vla.vla_kv_destroy(kv_b)
+    finally:
+        m.close()
+
+
+@pytest.mark.parametrize("max_ctx,ctx0", [(6144, 5000), (8192, 7000), (2368, 0)])
+def test_decode_long_and_empty_context_one_block(vla_lib, max_ctx, ctx0):
+    """Decode attention at the edges of its launch plans: three 128-key tiles per CTA
+    (max_ctx 6144), the shared-memory-ring kernel when a CTA's keys exceed three tiles
+    (max_ctx 8192), and the first token of an empty cache (one key in the whole context)."""
+    import torch
+    vla = vla_lib
+    s = synth.B7
+    m = Model(s, 1, 11, max_ctx)
+    try:
+        kv = vla.vla_kv_create(m.handle, 0, 1, max_ctx)
+        cache = oracle.KVCache([0], s.n_kv_heads, s.head_dim, max_ctx)
+        if ctx0:
+            kb, vb = synth.random_kv(ctx0, s, 11, 0)
+            kt, vt = kv_planes(vla, kv, 0, s, max_ctx)
+            kt[:, :ctx0].copy_(to_dev(kb))
+            vt[:, :ctx0].copy_(to_dev(vb))
+            cache.fill(0, oracle.bf16_to_f64(kb), oracle.bf16_to_f64(vb))
+            sync()
+            vla.vla_kv_set_length(kv, ctx0)
+        out = torch.empty((1, s.hidden), dtype=torch.bfloat16, device="cuda")
+        for t in range(2):
+            xt = synth.decode_hidden(t, s.hidden, 11)
+            ref = oracle.decode_step(oracle.bf16_to_f64(xt), m.weights64(), 0, 1, cache, s)
+            vla.vla_prefix_decode(m.handle, to_dev(xt), 0, 1, kv, out)
+            sync()
+            got = from_dev(out)
+            assert rel_l2(got, ref) < REL_L2_BLOCK, t
+            assert cos_sim(got, ref) > COS_FINAL, t
+        assert vla.vla_last_async_error(m.handle) == 0
+        assert vla.vla_kv_length(kv) == ctx0 + 2
+        vla.vla_kv_destroy(kv)
+    finally:
+        m.close()

@@ -309,6 +309,27 @@ def test_partition_identity_bit_exact():
             np.testing.assert_array_equal(c.v[l], c_full.v[l])
 
 
+def test_block_rows_equals_full_block_at_those_rows():
+    """The sampled-row evaluation used for full-size parity is the full block restricted to
+    some query rows: same outputs at those rows and the same cache entries, with and without
+    context before p0."""
+    s = Shape(32, 4, 2, 8, 40)
+    w = _stack(21, s, 1)[0]
+    x = np.random.default_rng(22).standard_normal((11, 32))
+    rows = [0, 3, 4, 10]
+    c = KVCache([0], 2, 8, 32)
+    full = oracle.block_forward(x, w, c, 0, s)
+    y, k, v = oracle.block_forward_rows(x, w, s, rows)
+    np.testing.assert_allclose(y, full[rows], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(k, c.k[0][:, :11], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(v, c.v[0][:, :11], rtol=1e-12, atol=1e-12)
+    x2 = np.random.default_rng(23).standard_normal((5, 32))
+    full2 = oracle.block_forward(x2, w, c, 0, s)  # positions 11..15 after the first call
+    y2, k2, _ = oracle.block_forward_rows(x2, w, s, [1, 4], p0=11, ctx_k=c.k[0], ctx_v=c.v[0])
+    np.testing.assert_allclose(y2, full2[[1, 4]], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(k2, c.k[0][:, 11:16], rtol=1e-12, atol=1e-12)
+
+
 def test_empty_range_returns_input():
     s = Shape(16, 2, 1, 8, 24)
     x = np.random.default_rng(14).standard_normal((3, 16))
