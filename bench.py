@@ -35,6 +35,8 @@ import synth  # noqa: E402
 METRIC = "prefix prefill tokens/s & % bf16 TC peak; decode µs/step & HBM GB/s (1 GB300)"
 WORKLOAD = "7b_prefix16_2304tok"
 DECODE_WORKLOAD = "7b_decode16_ctx2304"
+PIPELINE_WORKLOAD = "7b_pipeline32_3072tok"
+PIPELINE_SPLITS = (8, 16, 24)
 
 
 def _peaks():
@@ -226,13 +228,18 @@ def run_ours(args, dist: Dist):
     L = args.blocks or wl.prefix_layers
     M = wl.n_tokens
     D = s.hidden
+    pwl = synth.WORKLOADS[PIPELINE_WORKLOAD]
     dec_steps = dwl.decode_steps
-    max_ctx = max(M, dwl.prefill_ctx + dec_steps + 8)
+    pipeline_on = not args.no_pipeline and dist.world == 1
+    max_ctx = max(M, dwl.prefill_ctx + dec_steps + 8, pwl.n_tokens if pipeline_on else 0)
     seed = wl.seed
+    # the model holds every block of the 32-block stack when the pipeline phase runs (its
+    # splits go past block 16); the prefill and decode phases use blocks [0, L)
+    n_model = max(L, pwl.n_layers) if pipeline_on else L
 
     # ---- model: the prefix blocks (seeded synthetic weights), library-owned copies
     layers = []
-    for l in range(L):
+    for l in range(n_model):
         layers.append({k: to_dev(v, torch) for k, v in synth.layer_weights(s, seed, l).items()})
     cfg = vla.VlaConfig(hidden=D, n_heads=s.n_heads, n_kv_heads=s.n_kv_heads, head_dim=s.head_dim, ffn=s.ffn,
                         rms_eps=s.rms_eps, rope_base=s.rope_base, max_ctx=max_ctx)
@@ -338,10 +345,14 @@ def run_ours(args, dist: Dist):
         e2e = {"value": M * dist.world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": M * D * 2, "d2h_bytes_per_step": M * D * 2}
 
-    # ---- decode: 64 single-token steps against a 2304-position random context
+    # ---- decode: 64 single-token steps against a 2304-position random context, in a cache
+    # sized for the workload (2304 + 64 steps)
     decode = None
     if not args.no_decode:
         ctx0 = dwl.prefill_ctx
+        vla.vla_kv_destroy(kv)
+        max_ctx = ctx0 + dec_steps + 8
+        kv = vla.vla_kv_create(p, 0, L, max_ctx)
         for l in range(L):
             kb, vb = synth.random_kv(ctx0, s, dwl.seed, l)
             kp, vp = vla.vla_kv_data(kv, l)
@@ -396,6 +407,54 @@ def run_ours(args, dist: Dist):
                                "traffic": None},
                   "gpu_launches_per_step": dec_launches / (reps * dec_steps),
                   "stages_us_per_launch": {k: round(v[0] / v[1] * 1e3, 2) for k, v in dstages.items() if v[1]}}
+    # ---- pipeline (4 frames x 3072 tokens; prefix [0, k) of a 32-block stack for k = 8/16/24):
+    # frame t's boundary copy runs on the side stream under frame t+1's prefix
+    pipeline = None
+    if pipeline_on:
+        Mp = pwl.n_tokens
+        kvp = vla.vla_kv_create(p, 0, pwl.n_layers, Mp)
+        xs = [to_dev(synth.hidden_states(Mp, D, f, pwl.visual_tokens, pwl.visual_scale), torch)
+              for f in range(pwl.frames)]
+        hp = [torch.empty((Mp, D), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+        pp = [torch.empty((Mp, D), dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+        frame_flops = 2.0 * Mp * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                                  D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * Mp * Mp * s.head_dim * s.n_heads
+        splits = []
+        for k in PIPELINE_SPLITS:
+            def frames(copy: bool):
+                for f in range(pwl.frames):
+                    b = f & 1
+                    main.wait_event(done[b])
+                    vla.vla_kv_reset(kvp, main)
+                    vla.vla_prefix_prefill(p, xs[f], Mp, 0, k, kvp, hp[b], main)
+                    if copy:
+                        ready[b].record(main)
+                        vla.vla_boundary_to_host(hp[b], Mp, D, pp[b], side, ready[b], done[b])
+
+            frames(True)
+            torch.cuda.synchronize()
+            res = {}
+            for copy in (False, True):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(main)
+                frames(copy)
+                if copy:
+                    main.wait_event(done[(pwl.frames - 1) & 1])
+                e1.record(main)
+                torch.cuda.synchronize()
+                res[copy] = e0.elapsed_time(e1) / pwl.frames
+            assert torch.equal(pp[(pwl.frames - 1) & 1].view(torch.int16).cpu(),
+                               hp[(pwl.frames - 1) & 1].view(torch.int16).cpu())
+            tf = frame_flops * k / (res[False] * 1e-3) / 1e12
+            splits.append({"k": k, "ms_per_frame": res[True], "prefix_only_ms_per_frame": res[False],
+                           "copy_exposed_ms_per_frame": res[True] - res[False], "tflops": tf,
+                           "frac_of_peak": tf / bf16_sust, "boundary_bytes": Mp * D * 2})
+        assert vla.vla_last_async_error(p) == 0
+        vla.vla_kv_destroy(kvp)
+        pipeline = {"workload": PIPELINE_WORKLOAD, "frames": pwl.frames, "tokens": Mp, "blocks_total": pwl.n_layers,
+                    "note": "wall time per frame of the GPU prefix with the boundary copy to pinned host memory "
+                            "overlapped on a side stream, vs the prefix alone",
+                    "splits": splits}
     clock_info = clocks.stop()
 
     # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame
@@ -428,6 +487,7 @@ def run_ours(args, dist: Dist):
             "clocks": clock_info,
             "stages_ms_per_launch": {k: round(v[0] / v[1], 4) for k, v in stages.items() if v[1]},
             "decode": decode,
+            "pipeline": pipeline,
         }
         print(json.dumps(line), flush=True)
     vla.vla_kv_destroy(kv)
@@ -455,6 +515,7 @@ def main():
     ap.add_argument("--blocks", type=int, default=0, help="prefix depth (default: the workload's 16)")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-pipeline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -117,7 +117,6 @@ struct vla_prefix {
     // decode workspace
     float* dq = nullptr;
     bf16 *d_attn = nullptr, *d_xmid = nullptr, *d_m = nullptr;
-    int attn_tc = 0, attn_cs = 0, attn_cap = 0, attn_stages = 0;  // decode-attention plan
     unsigned* d_status = nullptr;
     int last_launches = 0;
     // measurement: event pairs around each kernel while timing is enabled
@@ -146,6 +145,8 @@ struct vla_kv {
     vla_prefix* p;
     int lb, le, max_ctx;
     size_t plane_elems;
+    // decode-attention launch plan for this cache's max_ctx (plan_decode_attention(_tc))
+    int attn_tc = 0, attn_cs = 0, attn_cap = 0, attn_stages = 0;
     bf16* data = nullptr;
     int* d_len = nullptr;
     std::vector<int> len;
@@ -305,11 +306,6 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         return VLA_ERR_OOM;
     }
     cudaError_t e = cudaMemset(p->d_status, 0, sizeof(unsigned));
-    if (e == cudaSuccess) {
-        p->attn_tc = vla::plan_decode_attention_tc(dh, H / Hkv, Hkv, T, &p->attn_cs, &p->attn_cap) ? 1 : 0;
-        if (!p->attn_tc)
-            e = vla::plan_decode_attention(dh, H / Hkv, Hkv, T, &p->attn_cs, &p->attn_cap, &p->attn_stages);
-    }
     if (e == cudaSuccess) e = vla::launch_rope_table(p->rope, T, dh, (double)cfg->rope_base, 0);
     p->layers.resize(layer_count);
     for (int l = 0; l < layer_count && e == cudaSuccess; ++l) {
@@ -364,6 +360,14 @@ vla_status vla_kv_create(vla_prefix* p, int layer_begin, int layer_end, int max_
     kv->le = layer_end;
     kv->max_ctx = max_ctx;
     kv->plane_elems = (size_t)p->cfg.n_kv_heads * max_ctx * p->cfg.head_dim;
+    const int dh = p->cfg.head_dim, Hkv = p->cfg.n_kv_heads, G = p->cfg.n_heads / Hkv;
+    kv->attn_tc = vla::plan_decode_attention_tc(dh, G, Hkv, max_ctx, &kv->attn_cs, &kv->attn_cap) ? 1 : 0;
+    if (!kv->attn_tc &&
+        vla::plan_decode_attention(dh, G, Hkv, max_ctx, &kv->attn_cs, &kv->attn_cap, &kv->attn_stages) != cudaSuccess) {
+        cudaGetLastError();
+        delete kv;
+        return VLA_ERR_UNSUPPORTED;
+    }
     const int nl = layer_end - layer_begin;
     kv->len.assign(nl, 0);
     if (!dmalloc(&kv->data, kv->plane_elems * 2 * nl) || !dmalloc(&kv->d_len, (size_t)nl)) {
@@ -572,7 +576,7 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
     vla::DecodeDims dims = {D, p->cfg.n_heads, p->cfg.n_kv_heads, p->cfg.head_dim, p->F_pad, kv->max_ctx,
                             p->cfg.rms_eps};
     vla::DecodeWork w = {p->dq,      p->d_attn,  p->d_xmid,  p->d_m,      p->rope,
-                         p->d_status, p->attn_tc, p->attn_cs, p->attn_cap, p->attn_stages};
+                         p->d_status, kv->attn_tc, kv->attn_cs, kv->attn_cap, kv->attn_stages};
     const int nl = layer_end - layer_begin;
     // enqueue the whole step on stream s, reading x_in and chaining through x_out
     auto enqueue = [&](const bf16* x_in, bf16* x_out, cudaStream_t s, const vla::StageHook& hook) {
