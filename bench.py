@@ -36,6 +36,7 @@ METRIC = "prefix prefill tokens/s & % bf16 TC peak; decode µs/step & HBM GB/s (
 WORKLOAD = "7b_prefix16_2304tok"
 DECODE_WORKLOAD = "7b_decode16_ctx2304"
 PIPELINE_WORKLOAD = "7b_pipeline32_3072tok"
+BLOCK_WORKLOAD = "7b_block_1024tok"
 PIPELINE_SPLITS = (8, 16, 24)
 
 
@@ -157,6 +158,23 @@ def oracle_prefill_time(n_tokens: int, seed: int = 0) -> tuple[float, int]:
     return time.perf_counter() - t0, os.cpu_count() or 1
 
 
+def oracle_decode_time(dwl) -> float:
+    """Seconds for the float64 oracle to run one decode step of one 7B-class block against the
+    decode workload's random context (weights and context converted outside the timed region)."""
+    import oracle
+    s = dwl.shape
+    if dwl.seed not in _ORACLE_W:
+        _ORACLE_W[dwl.seed] = oracle.LayerWeights.from_bf16(synth.layer_weights(s, dwl.seed, 0))
+    w = _ORACLE_W[dwl.seed]
+    kb, vb = synth.random_kv(dwl.prefill_ctx, s, dwl.seed, 0)
+    cache = oracle.KVCache([0], s.n_kv_heads, s.head_dim, dwl.prefill_ctx + 1)
+    cache.fill(0, oracle.bf16_to_f64(kb), oracle.bf16_to_f64(vb))
+    x = oracle.bf16_to_f64(synth.decode_hidden(0, s.hidden, dwl.seed))
+    t0 = time.perf_counter()
+    oracle.decode_step(x, {0: w}, 0, 1, cache, s)
+    return time.perf_counter() - t0
+
+
 def cpu_threads() -> int:
     for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
         if os.environ.get(v, "").isdigit():
@@ -211,6 +229,20 @@ def _traffic(kernel_key: str):
         return d["dram_bytes_per_launch"]
     except Exception:
         return None
+
+
+def _dec_gateup(dstages: dict, s, D: int) -> dict | None:
+    """Decode's largest kernel (gate/up GEMV + SwiGLU): weight bytes per launch over its
+    average launch time in the stage-timed pass (plain launches, no graph overlap)."""
+    ms, n = dstages.get("dec_gateup", (0.0, 0))
+    if not n:
+        return None
+    f_pad = (s.ffn + 255) // 256 * 256
+    nbytes = 2 * f_pad * D * 2
+    us = ms / n * 1e3
+    return {"kernel": "gemv_kernel<kGemvSwiGLU> (gate/up + SwiGLU)", "bytes_per_launch": nbytes,
+            "avg_launch_us": us, "achieved_gbs": nbytes / (us * 1e-6) / 1e9, "traffic": _traffic("dec_gateup"),
+            "timing": "stage-timed pass: plain launches, without the graph's programmatic overlap"}
 
 
 def run_ours(args, dist: Dist):
@@ -401,12 +433,50 @@ def run_ours(args, dist: Dist):
         dec_bytes = weight_bytes + kv_bytes
         dec_gbs = dec_bytes / (dec_us * 1e-6) / 1e9
         decode = {"workload": DECODE_WORKLOAD, "blocks": L, "us_per_step": dec_us, "bytes_per_step": dec_bytes,
+                  "attention_plan": vla.vla_kv_decode_plan(kv),
                   "hbm_gbs": dec_gbs,
                   "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": hbm_peak, "unit": "GB/s",
                                "frac": dec_gbs / hbm_peak, "peak_source": f"{peak_src} copy bandwidth",
                                "traffic": None},
+                  "dominant_kernel": _dec_gateup(dstages, s, D),
                   "gpu_launches_per_step": dec_launches / (reps * dec_steps),
                   "stages_us_per_launch": {k: round(v[0] / v[1] * 1e3, 2) for k, v in dstages.items() if v[1]}}
+    # ---- one 7B block over a 1024-token frame (768 visual rows at 2x scale + 256 text rows)
+    block1k = None
+    if not args.no_block1k:
+        bwl = synth.WORKLOADS[BLOCK_WORKLOAD]
+        Mb = bwl.n_tokens
+        xb1 = to_dev(synth.hidden_states(Mb, D, bwl.seed, bwl.visual_tokens, bwl.visual_scale), torch)
+        yb1 = torch.empty_like(xb1)
+        kv1 = vla.vla_kv_create(p, 0, 1, Mb)
+
+        def one_block():
+            vla.vla_kv_reset(kv1, main)
+            vla.vla_prefix_prefill(p, xb1, Mb, 0, 1, kv1, yb1, main)
+
+        for _ in range(args.warmup):
+            one_block()
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")  # > L2: weights re-read from HBM
+        times = []
+        for i in range(max(10, args.steps)):
+            flush.fill_(i & 0xFF)
+            b0, b1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            b0.record(main)
+            one_block()
+            b1.record(main)
+            torch.cuda.synchronize()
+            times.append(b0.elapsed_time(b1))
+        del flush
+        assert vla.vla_last_async_error(p) == 0
+        vla.vla_kv_destroy(kv1)
+        b_ms = statistics.median(times)
+        b_flops = 2.0 * Mb * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                              D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * Mb * Mb * s.head_dim * s.n_heads
+        block1k = {"workload": BLOCK_WORKLOAD, "tokens": Mb, "us_per_frame": b_ms * 1e3, "tokens_per_s": Mb / (b_ms * 1e-3),
+                   "tflops": b_flops / (b_ms * 1e-3) / 1e12, "frac_of_peak": b_flops / (b_ms * 1e-3) / 1e12 / bf16_burst,
+                   "peak": bf16_burst, "peak_source": f"{peak_src} bf16 burst (a single block timed alone)",
+                   "timing": "median of per-frame CUDA events, L2 flushed (256 MB write) before each frame"}
+
     # ---- pipeline (4 frames x 3072 tokens; prefix [0, k) of a 32-block stack for k = 8/16/24):
     # frame t's boundary copy runs on the side stream under frame t+1's prefix
     pipeline = None
@@ -459,6 +529,12 @@ def run_ours(args, dist: Dist):
 
     # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame
     cpu = None
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline and decode is not None:
+        t_dec = oracle_decode_time(dwl)
+        decode["cpu_baseline"] = {"value": t_dec * L * 1e6, "unit": "us/step", "cores": cpu_threads(),
+                                  "kind": "oracle",
+                                  "sample": f"one decode step of 1 of {L} blocks at context {dwl.prefill_ctx} "
+                                            f"({t_dec:.2f} s), extrapolated x{L}; float64 numpy oracle"}
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         t_cpu, _ = oracle_prefill_time(M)
         cpu = {"value": M / (t_cpu * L), "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
@@ -488,6 +564,7 @@ def run_ours(args, dist: Dist):
             "stages_ms_per_launch": {k: round(v[0] / v[1], 4) for k, v in stages.items() if v[1]},
             "decode": decode,
             "pipeline": pipeline,
+            "block_1024": block1k,
         }
         print(json.dumps(line), flush=True)
     vla.vla_kv_destroy(kv)
@@ -516,6 +593,7 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pipeline", action="store_true")
+    ap.add_argument("--no-block1k", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

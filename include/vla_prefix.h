@@ -100,9 +100,15 @@ vla_status vla_prefix_destroy(vla_prefix* p);
 /* KV cache for blocks [layer_begin, layer_end) of `p`, up to max_ctx positions per layer
  * (max_ctx <= cfg.max_ctx). Layout per layer: K plane then V plane, each
  * [n_kv_heads][max_ctx][head_dim] bf16; keys are stored after the rotary embedding.
- * Library-allocated, caller-owned (vla_kv_destroy). Lengths start at 0.
- * Errors: INVALID_ARG, RANGE, SHAPE (max_ctx), OOM. */
+ * Library-allocated, caller-owned (vla_kv_destroy). Lengths start at 0. The decode-attention
+ * launch plan for contexts up to max_ctx is fixed here (vla_kv_decode_plan).
+ * Errors: INVALID_ARG, RANGE, SHAPE (max_ctx), UNSUPPORTED (no attention plan), OOM. */
 vla_status vla_kv_create(vla_prefix* p, int layer_begin, int layer_end, int max_ctx, vla_kv** out);
+/* The decode-attention plan of this cache: *tensor_cores = 1 for the tcgen05 kernel (head_dim
+ * 128), 0 for the CUDA-core kernel; *cluster_size = CTAs per KV head (key splits, one thread-
+ * block cluster); *keys_per_cta = keys one CTA holds in shared memory (tcgen05: its whole key
+ * range; CUDA-core: one stage of its ring). Any output pointer may be NULL. Errors: INVALID_ARG. */
+vla_status vla_kv_decode_plan(const vla_kv* kv, int* tensor_cores, int* cluster_size, int* keys_per_cta);
 vla_status vla_kv_destroy(vla_kv* kv);
 /* Sets every layer's length to 0 (contents are left as they are). Ordered on `stream`. */
 vla_status vla_kv_reset(vla_kv* kv, vla_stream stream);
@@ -159,7 +165,7 @@ int vla_last_launch_count(const vla_prefix* p);
  * summed kernel time in milliseconds and the number of launches since the last read, then
  * clears them. Arrays have n_stages entries (VLA_STAGE_COUNT covers all). */
 enum {
-    VLA_STAGE_ROWSTAT = 0,      /* RMSNorm 1/rms rows (prefill)                  */
+    VLA_STAGE_ROWSTAT = 0,      /* RMSNorm row statistics of a range's input     */
     VLA_STAGE_GEMM_QKV = 1,     /* QKV projection + RoPE + KV write (prefill)   */
     VLA_STAGE_ATTN = 2,         /* causal GQA attention (prefill)               */
     VLA_STAGE_GEMM_O = 3,       /* output projection + residual (prefill)       */

@@ -17,7 +17,7 @@ from ._build import build as _build_lib
 __all__ = [
     "build", "load", "VlaError", "VlaConfig", "VlaLayerWeights",
     "vla_prefix_create", "vla_prefix_destroy", "vla_kv_create", "vla_kv_destroy", "vla_kv_reset",
-    "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_set_length", "vla_prefix_prefill",
+    "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
     "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
     "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "STATUS", "STAGES",
@@ -75,6 +75,7 @@ def load():
         "vla_prefix_destroy": ([P], I),
         "vla_kv_create": ([P, I, I, I, ctypes.POINTER(P)], I),
         "vla_kv_destroy": ([P], I),
+        "vla_kv_decode_plan": ([P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)], I),
         "vla_kv_reset": ([P, V], I),
         "vla_kv_length": ([P], I),
         "vla_kv_layer_length": ([P, I], I),
@@ -178,6 +179,14 @@ def vla_kv_length(kv) -> int:
 
 def vla_kv_layer_length(kv, layer: int) -> int:
     return load().vla_kv_layer_length(kv, layer)
+
+
+def vla_kv_decode_plan(kv) -> dict:
+    """The cache's decode-attention launch plan: tensor_cores, cluster_size, keys_per_cta."""
+    tc, cs, keys = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(load().vla_kv_decode_plan(kv, ctypes.byref(tc), ctypes.byref(cs), ctypes.byref(keys)),
+           "vla_kv_decode_plan")
+    return {"tensor_cores": tc.value, "cluster_size": cs.value, "keys_per_cta": keys.value}
 
 
 def vla_kv_data(kv, layer: int):

@@ -120,6 +120,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem_slot;
+    pdl_wait();  // Q, K and V are the previous kernel's output
+    pdl_trigger();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -352,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int DH>
-cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream) {
+cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream, bool pdl) {
     using C = AttnCfg<DH>;
     static bool attr_set = false;
     if (!attr_set) {
@@ -378,16 +380,15 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
     a.out = p.out;
     a.status = status;
     dim3 grid((p.M + kBM - 1) / kBM, p.H);
-    attn_prefill_tc_kernel<DH><<<grid, kThreads, C::SMEM, stream>>>(tq, tk, tv, a);
-    return cudaGetLastError();
+    return launch_ex(attn_prefill_tc_kernel<DH>, grid, dim3(kThreads), C::SMEM, stream, pdl, tq, tk, tv, a);
 }
 
 }  // namespace
 
-cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream) {
+cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream, bool pdl) {
     if (p.M <= 0) return cudaSuccess;
-    if (p.head_dim == 128) return launch_dh<128>(p, status, stream);
-    if (p.head_dim == 64) return launch_dh<64>(p, status, stream);
+    if (p.head_dim == 128) return launch_dh<128>(p, status, stream, pdl);
+    if (p.head_dim == 64) return launch_dh<64>(p, status, stream, pdl);
     return cudaErrorInvalidValue;
 }
 

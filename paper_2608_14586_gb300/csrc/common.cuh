@@ -265,6 +265,24 @@ VLA_DEV float ld_dsmem_f32(const float* local, uint32_t rank) {
     return v;
 }
 
+// Host side: launch with programmatic stream serialization when `pdl` is set, so the kernel
+// may start while the previous kernel in the stream drains. Such a kernel must execute
+// pdl_wait() before reading anything an earlier kernel wrote, and write nothing before it.
+template <typename Kern, typename... Args>
+inline cudaError_t launch_ex(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 VLA_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 VLA_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

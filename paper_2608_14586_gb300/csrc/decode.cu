@@ -435,24 +435,6 @@ __global__ void advance_lengths_kernel(int* d_len, int count) {
     if (i < count) d_len[i] += 1;
 }
 
-// Launch with programmatic stream serialization when `pdl` is set: the kernel may start while
-// the previous kernel in the stream drains; every decode kernel reads data produced by its
-// predecessors only after griddepcontrol.wait and writes nothing before it.
-template <typename Kern, typename... Args>
-cudaError_t launch_kernel(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl, Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, kern, args...);
-}
-
 template <int MODE>
 cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
     const size_t smem = (size_t)p.K * 2;
@@ -466,7 +448,7 @@ cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s, bool p
     int grid = 2 * num_sms;
     const int gmax = (warps_needed + 7) / 8;
     if (grid > gmax) grid = gmax;
-    return launch_kernel(gemv_kernel<MODE>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
+    return launch_ex(gemv_kernel<MODE>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
 }
 
 template <int DH, int G>

@@ -7,26 +7,28 @@ namespace vla {
 
 namespace {
 
-// One warp per row: rinv = 1 / sqrt(mean(x^2) + eps), fp32 sum of squares, 16-byte loads.
-__global__ void rowstat_kernel(const bf16* __restrict__ x, int M, int D, int ld, float eps,
-                               float* __restrict__ rinv) {
-    const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (row >= M) return;
-    const bf16* xr = x + (size_t)row * ld;
+// One thread per (row, 256-column chunk): fp32 sum of squares over the chunk's columns in
+// order, exactly as the residual GEMM epilogue accumulates its stored outputs.
+__global__ void row_sumsq_kernel(const bf16* __restrict__ x, int M, int chunks, int ld, float* __restrict__ ss) {
+    const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    pdl_wait();  // x is the previous kernel's output
+    pdl_trigger();
+    if (i >= (long long)M * chunks) return;
+    const int row = (int)(i / chunks), t = (int)(i % chunks);
+    const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * ld + t * 256);
     float acc = 0.f;
-    for (int c = lane * 8; c < D; c += 32 * 8) {
-        const uint4 v = *reinterpret_cast<const uint4*>(xr + c);
+#pragma unroll 4
+    for (int c = 0; c < 32; ++c) {
+        const uint4 v = xr[c];
         const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float a = bf16_lo(w[i]), b = bf16_hi(w[i]);
+        for (int k = 0; k < 4; ++k) {
+            const float a = bf16_lo(w[k]), b = bf16_hi(w[k]);
             acc = fmaf(a, a, acc);
             acc = fmaf(b, b, acc);
         }
     }
-    acc = warp_sum(acc);
-    if (lane == 0) rinv[row] = 1.0f / sqrtf(acc / (float)D + eps);
+    ss[i] = acc;
 }
 
 // table[pos][j] = (cos, sin)(pos * base^(-2j/dh)), angles in float64
@@ -95,12 +97,12 @@ __global__ void set_lengths_kernel(int* d_len, int count, int value) {
 
 }  // namespace
 
-cudaError_t launch_rowstat(const bf16* x, int M, int D, int ld, float eps, float* rinv, cudaStream_t stream) {
+cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl) {
     if (M <= 0) return cudaSuccess;
-    const int rows_per_block = 8;
-    rowstat_kernel<<<(M + rows_per_block - 1) / rows_per_block, rows_per_block * 32, 0, stream>>>(x, M, D, ld, eps,
-                                                                                                  rinv);
-    return cudaGetLastError();
+    const int chunks = D / 256;
+    const long long n = (long long)M * chunks;
+    return launch_ex(row_sumsq_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, stream, pdl, x, M, chunks, ld,
+                     ss);
 }
 
 cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream) {

@@ -59,9 +59,18 @@ VLA_DEV void store_bf16x32(bf16* dst, const float (&v)[32]) {
 // Epilogues. Each thread owns one output row (TMEM lane); all 32 lanes of a warp execute
 // every tcgen05.ld; stores are masked per row / column.
 // ---------------------------------------------------------------------------------------
+// 1/rms of an input row from its 256-column partial sums of squares (chunk order)
+VLA_DEV float row_rinv(const EpiParams& ep, int row) {
+    const float* ps = ep.ss_in + (size_t)row * ep.ss_chunks;
+    float t = 0.f;
+    for (int c = 0; c < ep.ss_chunks; ++c) t += ps[c];
+    return 1.0f / sqrtf(t / (float)ep.norm_dim + ep.eps);
+}
+
 template <int BN>
 VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const bool row_ok = row < ep.M;
+    float ss = 0.f;  // sum of squares of the stored outputs, columns in order
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
         uint32_t r[32];
@@ -89,6 +98,13 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
                 }
             }
             store_bf16x32(op, v);
+            if (ep.ss_out) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float r = __bfloat162float(__float2bfloat16_rn(v[i]));
+                    ss = fmaf(r, r, ss);
+                }
+            }
         } else {
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -100,12 +116,14 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
             }
         }
     }
+    // the row statistics of the next RMSNorm (BN = 256: one partial per 256-column chunk)
+    if (ep.ss_out && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_chunks + n0 / 256] = ss;
 }
 
 template <int BN>
 VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const bool row_ok = row < ep.M;
-    const float s = row_ok ? ep.rinv[row] : 0.f;
+    const float s = row_ok ? row_rinv(ep, row) : 0.f;
     const int pos = ep.pos0 + row;
     const int dh = ep.head_dim;
     const int half = dh >> 1;
@@ -162,7 +180,7 @@ template <int BN>
 VLA_DEV void epi_swiglu(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     constexpr int HALF = BN / 2;
     const bool row_ok = row < ep.M;
-    const float s = row_ok ? ep.rinv[row] : 0.f;
+    const float s = row_ok ? row_rinv(ep, row) : 0.f;
     const int f0 = (n0 / BN) * HALF;
 #pragma unroll 1
     for (int c = 0; c < HALF; c += 32) {
@@ -253,6 +271,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t phase = 0;
             uint32_t issued = 0, issued_phase = 0;  // per-stage bit masks of loads in flight
             bool ok = true;
+            // The weight tiles (B) do not depend on the previous kernel: under programmatic
+            // dependent launch the first ring's worth of them is requested before the wait,
+            // while the previous kernel drains. Activations (A) only after it.
+            const int pre = (blockIdx.x < num_tiles) ? min(STAGES, num_kb) : 0;
+            for (int kb = 0; kb < pre; ++kb) {
+                mbar_arrive_expect_tx(&full[kb], C::STAGE_BYTES);
+                tma_load_2d(sB + kb * C::B_BYTES, &tmB, &full[kb], kb * kBK, (blockIdx.x / num_m) * BN);
+                issued |= 1u << kb;
+            }
+            pdl_wait();
+            pdl_trigger();
+            bool first = true;
             for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
                 const int m0 = (tile % num_m) * kBM;
                 const int n0 = (tile / num_m) * BN;
@@ -261,9 +291,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
-                    tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
-                    tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * kBK, n0);
+                    if (first && kb < pre) {  // B of this stage is already in flight
+                        tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
+                    } else {
+                        mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+                        tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
+                        tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * kBK, n0);
+                    }
                     issued |= 1u << stage;
                     issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
                     if (++stage == STAGES) {
@@ -271,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         phase ^= 1u;
                     }
                 }
+                first = false;
             }
             if (!ok) {
                 s_abort = 1;
@@ -281,6 +316,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else if (warp == 1) {
+        pdl_wait();
+        pdl_trigger();
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
             int stage = 0;
@@ -327,6 +364,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ---------------- epilogue (warps 2..5) ----------------
+        pdl_wait();  // the epilogue reads 1/rms and the residual written by earlier kernels
+        pdl_trigger();
         const int quarter = warp & 3;  // TMEM lanes [32*quarter, 32*quarter + 32)
         int it = 0;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
@@ -366,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K, const EpiParams& ep,
-                       int num_sms, cudaStream_t stream) {
+                       int num_sms, cudaStream_t stream, bool pdl) {
     using C = GemmCfg<BN>;
     static bool attr_set = false;
     auto kern = gemm_bf16_tcgen05<BN, EPI>;
@@ -377,28 +416,29 @@ cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N,
     }
     const int tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
     const int grid = tiles < num_sms ? tiles : num_sms;
-    kern<<<grid, kThreads, C::SMEM_BYTES, stream>>>(A, B, M, N, K, ep);
-    return cudaGetLastError();
+    return launch_ex(kern, dim3(grid), dim3(kThreads), C::SMEM_BYTES, stream, pdl, A, B, M, N, K, ep);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
-                        const EpiParams& ep, int num_sms, cudaStream_t stream) {
+                        const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl) {
     if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
     if (bn == 256) {
         switch (mode) {
             case kEpiPlain:
-            case kEpiResid: return launch_one<256, kEpiResid>(A, B, M, N, K, ep, num_sms, stream);
-            case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream);
-            case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiResid: return launch_one<256, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream, pdl);
         }
     } else if (bn == 128) {
         switch (mode) {
             case kEpiPlain:
-            case kEpiResid: return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream);
-            case kEpiQKV: return launch_one<128, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream);
-            case kEpiSwiGLU: return launch_one<128, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream);
+            case kEpiResid:
+                if (ep.ss_out) return cudaErrorInvalidValue;  // row partials are per 256 columns
+                return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiQKV: return launch_one<128, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiSwiGLU: return cudaErrorInvalidValue;  // gate/up rows are interleaved for BN = 256
         }
     }
     return cudaErrorInvalidValue;

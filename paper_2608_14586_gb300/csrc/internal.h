@@ -16,8 +16,8 @@ using bf16 = __nv_bfloat16;
 enum EpiMode : int {
     kEpiPlain = 0,   // out = bf16(acc)
     kEpiResid = 1,   // out = bf16(resid + acc)                       (O / down projections)
-    kEpiQKV = 2,     // acc * rinv -> RoPE(q, k); q -> out, k/v -> KV cache (QKV projection)
-    kEpiSwiGLU = 3,  // gate/up tiles interleaved by 128 columns: out = silu(g*rinv) * (u*rinv)
+    kEpiQKV = 2,     // acc / rms -> RoPE(q, k); q -> out, k/v -> KV cache (QKV projection)
+    kEpiSwiGLU = 3,  // gate/up tiles interleaved by 128 columns: out = silu(g/rms) * (u/rms)
 };
 
 struct EpiParams {
@@ -26,7 +26,15 @@ struct EpiParams {
     int ld_out;
     const bf16* resid;
     int ld_resid;
-    const float* rinv;  // per-row 1/rms
+    // RMSNorm of the GEMM's input rows: 1/rms = 1/sqrt(sum_t ss_in[row][t] / D + eps), the
+    // partial sums of squares over 256-column chunks added in chunk order (kEpiQKV, kEpiSwiGLU)
+    const float* ss_in;
+    int ss_chunks;  // D / 256
+    int norm_dim;   // D
+    float eps;
+    // kEpiResid: per-row partial sums of squares of the stored (bf16) outputs of this tile's
+    // 256 columns -> ss_out[row][n0 / 256] (nullptr: not wanted)
+    float* ss_out;
     // QKV epilogue
     bf16* kcache;        // layer base, [n_kv_heads][max_ctx][head_dim]
     bf16* vcache;
@@ -46,8 +54,10 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint6
                        uint64_t plane_stride, uint32_t box_rows);
 
 // Launch: BN in {128, 256}. Returns a cudaError_t of the launch.
+// pdl: programmatic dependent launch (the CTA prologue and the first weight-tile loads may
+// overlap the previous kernel; A and everything the epilogue reads come after the wait).
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
-                        const EpiParams& ep, int num_sms, cudaStream_t stream);
+                        const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl = false);
 
 // ---------------------------------------------------------------------------------------
 // Prefill attention (causal GQA, flash-style online softmax, attention_tc.cu)
@@ -63,13 +73,16 @@ struct AttnPrefillParams {
     float scale_log2;  // log2(e) / sqrt(dh)
 };
 // tcgen05 kernel (S and O in tensor memory); `status` receives a timeout code
-cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream);
+cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream,
+                                   bool pdl = false);
 
 // ---------------------------------------------------------------------------------------
 // Elementwise / setup kernels
 // ---------------------------------------------------------------------------------------
-// rinv[i] = 1 / sqrt(mean_d x[i,d]^2 + eps)
-cudaError_t launch_rowstat(const bf16* x, int M, int D, int ld, float eps, float* rinv, cudaStream_t stream);
+// ss[i][t] = sum over columns [256t, 256t+256) of x[i][c]^2 (fp32, columns in order): the same
+// partial sums the residual GEMM epilogue writes for its output, so a block gets bit-identical
+// row statistics whether its input came from the previous block or from the caller.
+cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl = false);
 
 // cos/sin table [max_ctx][dh/2] from float64 angles pos * base^(-2j/dh)
 cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream);

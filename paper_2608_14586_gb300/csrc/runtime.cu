@@ -1,17 +1,18 @@
 // C-ABI runtime of the LLM-prefix library (include/vla_prefix.h, include/vla_ops.h).
 //
 // Per block l of a prefill over [layer_begin, layer_end), on the caller's stream:
-//   rowstat(x)                         1/rms per token                      (RMSNorm, part 1)
-//   GEMM  x * Wqkv^T   [kEpiQKV]       1/rms scale, RoPE, q -> workspace,   (RMSNorm part 2,
-//                                      post-RoPE k and v -> KV cache         projection, RoPE)
+//   row_sumsq(x)        (first block)  sum of x^2 per 256-column chunk      (RMSNorm statistics)
+//   GEMM  x * Wqkv^T   [kEpiQKV]       1/rms scale, RoPE, q -> workspace,   (RMSNorm, projection,
+//                                      post-RoPE k and v -> KV cache         RoPE, KV write)
 //   attention(q, K, V)                 causal GQA over cache [0, p0 + M)
-//   GEMM  o * Wo^T     [kEpiResid]     x_mid = x + o Wo^T
-//   rowstat(x_mid)
-//   GEMM  x_mid * Wgu^T [kEpiSwiGLU]   m = silu(gate) * up
-//   GEMM  m * Wd^T     [kEpiResid]     x_out = x_mid + m Wd^T -> hidden_out
-// Block b reads hidden_in; later blocks work in place in hidden_out, so the range needs one
-// extra [M, D] buffer (x_mid). hidden_out after the last block is h^(layer_end) (Eq. 5).
-// Decode runs the same stages as GEMVs (decode.cu), replayed as a CUDA graph per step.
+//   GEMM  o * Wo^T     [kEpiResid]     x_mid = x + o Wo^T, and x_mid's row statistics
+//   GEMM  x_mid * Wgu^T [kEpiSwiGLU]   1/rms scale, m = silu(gate) * up
+//   GEMM  m * Wd^T     [kEpiResid]     x_out = x_mid + m Wd^T -> hidden_out, and its row
+//                                      statistics for block l+1
+// Every kernel after the first is launched with programmatic dependent launch. Block b reads
+// hidden_in; later blocks work in place in hidden_out, so the range needs one extra [M, D]
+// buffer (x_mid). hidden_out after the last block is h^(layer_end) (Eq. 5). Decode runs the
+// same stages as GEMVs (decode.cu, decode_attn_tc.cu), replayed as a CUDA graph per step.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -87,7 +88,16 @@ static int device_sm_count() {
 
 namespace {
 
-constexpr int kBN = 256;  // N tile of every prefill GEMM
+constexpr int kBN = 256;  // N tile of the prefill GEMMs (the QKV GEMM may use 128, below)
+
+// 256 or 128: the N tile that finishes a GEMM of M x N output in fewer SM waves, counting a
+// 128-wide tile as 0.55 of a 256-wide one (half the MMAs plus fixed per-tile cost).
+int gemm_tile_width(int M, int N, int sms) {
+    const int m_tiles = (M + 127) / 128;
+    const int w256 = (m_tiles * ((N + 255) / 256) + sms - 1) / sms;
+    const int w128 = (m_tiles * ((N + 127) / 128) + sms - 1) / sms;
+    return (0.55 * w128 < 1.0 * w256) ? 128 : 256;
+}
 
 // A decode step is ~6 kernels per block (~97 for 16 blocks), each only a few to a few tens
 // of microseconds long, so host launch cost would dominate. The step is captured once per
@@ -99,6 +109,7 @@ constexpr int kMaxDecodeGraphs = 8;
 struct LayerDev {
     bf16 *w_qkv, *w_o, *w_gu, *w_d;
     CUtensorMap tm_qkv, tm_o, tm_gu, tm_d;
+    CUtensorMap tm_qkv128;  // W_qkv with 128-row boxes (QKV GEMM with 128-column tiles)
 };
 
 }  // namespace
@@ -113,7 +124,7 @@ struct vla_prefix {
     float2* rope = nullptr;
     // prefill workspace, sized for cfg.max_ctx tokens
     bf16 *ws_q = nullptr, *ws_attn = nullptr, *ws_xmid = nullptr, *ws_m = nullptr;
-    float* ws_rinv = nullptr;
+    float *ws_ss_x = nullptr, *ws_ss_mid = nullptr;  // [max_ctx][D/256] row sums of squares
     // decode workspace
     float* dq = nullptr;
     bf16 *d_attn = nullptr, *d_xmid = nullptr, *d_m = nullptr;
@@ -171,7 +182,8 @@ void free_prefix(vla_prefix* p) {
     cudaFree(p->ws_attn);
     cudaFree(p->ws_xmid);
     cudaFree(p->ws_m);
-    cudaFree(p->ws_rinv);
+    cudaFree(p->ws_ss_x);
+    cudaFree(p->ws_ss_mid);
     cudaFree(p->dq);
     cudaFree(p->d_attn);
     cudaFree(p->d_xmid);
@@ -296,7 +308,8 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
     bool ok = dmalloc(&p->weight_pool, per_layer * layer_count) && dmalloc(&p->rope, (size_t)T * dh / 2) &&
               dmalloc(&p->ws_q, (size_t)T * p->qc) && dmalloc(&p->ws_attn, (size_t)T * p->qc) &&
               dmalloc(&p->ws_xmid, (size_t)T * D) && dmalloc(&p->ws_m, (size_t)T * p->F_pad) &&
-              dmalloc(&p->ws_rinv, (size_t)T) && dmalloc(&p->dq, (size_t)p->qc) &&
+              dmalloc(&p->ws_ss_x, (size_t)T * (D / 256)) &&
+              dmalloc(&p->ws_ss_mid, (size_t)T * (D / 256)) && dmalloc(&p->dq, (size_t)p->qc) &&
               dmalloc(&p->d_attn, (size_t)p->qc) && dmalloc(&p->d_xmid, (size_t)D) &&
               dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1) &&
               dmalloc(&p->d_xin, (size_t)D) && dmalloc(&p->d_xout, (size_t)D);
@@ -323,6 +336,7 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         e = vla::launch_repack(s, d, D, H, Hkv, dh, cfg->ffn, p->F_pad, 0);
         if (e != cudaSuccess) break;
         if (!vla::make_tmap_bf16(&ld.tm_qkv, ld.w_qkv, p->qkv_n, D, D, kBN) ||
+            !vla::make_tmap_bf16(&ld.tm_qkv128, ld.w_qkv, p->qkv_n, D, D, 128) ||
             !vla::make_tmap_bf16(&ld.tm_o, ld.w_o, D, p->qc, p->qc, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_gu, ld.w_gu, 2 * p->F_pad, D, D, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_d, ld.w_d, D, p->F_pad, p->F_pad, kBN)) {
@@ -421,6 +435,14 @@ int vla_kv_length(const vla_kv* kv) {
     return m;
 }
 
+vla_status vla_kv_decode_plan(const vla_kv* kv, int* tensor_cores, int* cluster_size, int* keys_per_cta) {
+    if (!kv) return VLA_ERR_INVALID_ARG;
+    if (tensor_cores) *tensor_cores = kv->attn_tc;
+    if (cluster_size) *cluster_size = kv->attn_cs;
+    if (keys_per_cta) *keys_per_cta = kv->attn_cap;
+    return VLA_OK;
+}
+
 int vla_kv_layer_length(const vla_kv* kv, int layer) {
     if (!kv || layer < kv->lb || layer >= kv->le) return -1;
     return kv->len[layer - kv->lb];
@@ -460,21 +482,39 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
     int launches = 0;
     cudaError_t e = cudaSuccess;
     p->cur_stream = stream;
+    // Programmatic dependent launch for every kernel after the call's first, except the ones
+    // being timed (their start event must precede the whole kernel).
+    bool first_launch = true;
+    auto pdl = [&](int stage) {
+        const bool r = !first_launch && !((p->timing >> stage) & 1u);
+        first_launch = false;
+        return r;
+    };
+    // QKV tile width: 128 columns when that needs fewer 256-column-equivalent waves (short
+    // frames: at M = 1024 the 256-wide grid is 1.26 waves of 152 SMs, the 128-wide one 2.5)
+    const int qkv_bn = gemm_tile_width(M, p->qkv_n, p->num_sms);
     for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
         const LayerDev& ld = p->layers[l];
         const bf16* x = (l == layer_begin) ? (const bf16*)hidden_in : (const bf16*)hidden_out;
         const CUtensorMap& tm_x = (l == layer_begin) ? tm_in : tm_out;
-        // RMSNorm row statistics + QKV projection + RoPE + KV write
-        stage_mark(p, VLA_STAGE_ROWSTAT, true);
-        e = vla::launch_rowstat(x, M, D, D, eps, p->ws_rinv, stream);
-        stage_mark(p, VLA_STAGE_ROWSTAT, false);
-        if (e != cudaSuccess) break;
+        // RMSNorm row statistics of the range's input (later blocks get them from the previous
+        // block's down-projection epilogue) + QKV projection + RoPE + KV write
+        if (l == layer_begin) {
+            stage_mark(p, VLA_STAGE_ROWSTAT, true);
+            e = vla::launch_row_sumsq(x, M, D, D, p->ws_ss_x, stream, pdl(VLA_STAGE_ROWSTAT));
+            stage_mark(p, VLA_STAGE_ROWSTAT, false);
+            if (e != cudaSuccess) break;
+            ++launches;
+        }
         vla::EpiParams ep = {};
         ep.M = M;
         ep.N = p->qkv_n;
         ep.out = p->ws_q;
         ep.ld_out = p->qc;
-        ep.rinv = p->ws_rinv;
+        ep.ss_in = p->ws_ss_x;
+        ep.ss_chunks = D / 256;
+        ep.norm_dim = D;
+        ep.eps = eps;
         ep.kcache = kv->k_plane(l);
         ep.vcache = kv->v_plane(l);
         ep.rope = p->rope;
@@ -485,7 +525,8 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ep.kv_cols = p->kvc;
         ep.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_QKV, true);
-        e = vla::launch_gemm(vla::kEpiQKV, kBN, tm_x, ld.tm_qkv, M, p->qkv_n, D, ep, p->num_sms, stream);
+        e = vla::launch_gemm(vla::kEpiQKV, qkv_bn, tm_x, qkv_bn == 128 ? ld.tm_qkv128 : ld.tm_qkv, M, p->qkv_n, D, ep,
+                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_QKV));
         stage_mark(p, VLA_STAGE_GEMM_QKV, false);
         if (e != cudaSuccess) break;
         // causal GQA attention over the cache
@@ -504,7 +545,7 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ap.pos0 = p0;
         ap.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)p->cfg.head_dim));
         stage_mark(p, VLA_STAGE_ATTN, true);
-        e = vla::launch_attn_prefill_tc(ap, p->d_status, stream);
+        e = vla::launch_attn_prefill_tc(ap, p->d_status, stream, pdl(VLA_STAGE_ATTN));
         stage_mark(p, VLA_STAGE_ATTN, false);
         if (e != cudaSuccess) break;
         // output projection + residual
@@ -515,25 +556,28 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         eo.ld_out = D;
         eo.resid = x;
         eo.ld_resid = D;
+        eo.ss_out = p->ws_ss_mid;
+        eo.ss_chunks = D / 256;
         eo.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_O, true);
-        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_attn, ld.tm_o, M, D, p->qc, eo, p->num_sms, stream);
+        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_attn, ld.tm_o, M, D, p->qc, eo, p->num_sms, stream,
+                             pdl(VLA_STAGE_GEMM_O));
         stage_mark(p, VLA_STAGE_GEMM_O, false);
         if (e != cudaSuccess) break;
-        // RMSNorm + gate/up + SwiGLU
-        stage_mark(p, VLA_STAGE_ROWSTAT, true);
-        e = vla::launch_rowstat(p->ws_xmid, M, D, D, eps, p->ws_rinv, stream);
-        stage_mark(p, VLA_STAGE_ROWSTAT, false);
-        if (e != cudaSuccess) break;
+        // RMSNorm (row statistics from the O epilogue) + gate/up + SwiGLU
         vla::EpiParams eg = {};
         eg.M = M;
         eg.N = 2 * p->F_pad;
         eg.out = p->ws_m;
         eg.ld_out = p->F_pad;
-        eg.rinv = p->ws_rinv;
+        eg.ss_in = p->ws_ss_mid;
+        eg.ss_chunks = D / 256;
+        eg.norm_dim = D;
+        eg.eps = eps;
         eg.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_GATEUP, true);
-        e = vla::launch_gemm(vla::kEpiSwiGLU, kBN, tm_xmid, ld.tm_gu, M, 2 * p->F_pad, D, eg, p->num_sms, stream);
+        e = vla::launch_gemm(vla::kEpiSwiGLU, kBN, tm_xmid, ld.tm_gu, M, 2 * p->F_pad, D, eg, p->num_sms, stream,
+                             pdl(VLA_STAGE_GEMM_GATEUP));
         stage_mark(p, VLA_STAGE_GEMM_GATEUP, false);
         if (e != cudaSuccess) break;
         // down projection + residual -> hidden_out
@@ -544,11 +588,14 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ed.ld_out = D;
         ed.resid = p->ws_xmid;
         ed.ld_resid = D;
+        ed.ss_out = (l + 1 < layer_end) ? p->ws_ss_x : nullptr;  // the next block's row statistics
+        ed.ss_chunks = D / 256;
         ed.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_DOWN, true);
-        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_m, ld.tm_d, M, D, p->F_pad, ed, p->num_sms, stream);
+        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_m, ld.tm_d, M, D, p->F_pad, ed, p->num_sms, stream,
+                             pdl(VLA_STAGE_GEMM_DOWN));
         stage_mark(p, VLA_STAGE_GEMM_DOWN, false);
-        launches += 7;
+        launches += 5;
     }
     if (e != cudaSuccess) return VLA_ERR_CUDA;
     for (int l = layer_begin; l < layer_end; ++l) kv->len[l - kv->lb] = p0 + M;
