@@ -35,17 +35,6 @@ constexpr uint32_t kTmemCols = 64;                  // S^T tiles at [16t, 16t+16
 constexpr uint32_t kOCol = 48;
 constexpr int kMaxCs = 16;
 
-VLA_DEV void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];\n\t"
-        "tcgen05.wait::ld.sync.aligned;\n"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-}
-
 // byte offset of (row, 16-byte chunk j) inside a 128-byte-swizzled tile of 128-byte rows
 VLA_DEV uint32_t sw128_off(int row, int j) { return (uint32_t)row * 128u + ((uint32_t)(j ^ (row & 7)) << 4); }
 
