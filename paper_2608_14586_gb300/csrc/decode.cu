@@ -574,7 +574,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
                                 bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook, bool pdl_first) {
     cudaError_t e;
     // stage timing records events between the launches: launch those fully serialized
-    const bool pdl = hook.fn == nullptr;
+    const bool pdl = hook.fn == nullptr && pdl_enabled();
     pdl_first = pdl_first && pdl;
     const int qc = d.H * d.dh, kvc = d.Hkv * d.dh;
     // 1. RMSNorm + QKV + RoPE + KV append

@@ -53,6 +53,10 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t planes,
                        uint64_t plane_stride, uint32_t box_rows);
 
+// Programmatic dependent launch is used unless the environment sets VLA_NO_PDL (read once;
+// for profilers and debuggers that serialise kernels anyway).
+bool pdl_enabled();
+
 // Launch: BN in {128, 256}. Returns a cudaError_t of the launch.
 // pdl: programmatic dependent launch (the CTA prologue and the first weight-tile loads may
 // overlap the previous kernel; A and everything the epilogue reads come after the wait).

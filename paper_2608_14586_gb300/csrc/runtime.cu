@@ -19,6 +19,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -75,6 +76,11 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint6
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+bool pdl_enabled() {
+    static const bool on = std::getenv("VLA_NO_PDL") == nullptr;
+    return on;
 }
 
 static int device_sm_count() {
@@ -486,7 +492,7 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
     // being timed (their start event must precede the whole kernel).
     bool first_launch = true;
     auto pdl = [&](int stage) {
-        const bool r = !first_launch && !((p->timing >> stage) & 1u);
+        const bool r = !first_launch && !((p->timing >> stage) & 1u) && vla::pdl_enabled();
         first_launch = false;
         return r;
     };
