@@ -171,7 +171,7 @@ enum {
     VLA_STAGE_GEMM_O = 3,       /* output projection + residual (prefill)       */
     VLA_STAGE_GEMM_GATEUP = 4,  /* gate/up projection + SwiGLU (prefill)        */
     VLA_STAGE_GEMM_DOWN = 5,    /* down projection + residual (prefill)         */
-    VLA_STAGE_KV_LEN = 6,       /* KV length update                              */
+    VLA_STAGE_KV_LEN = 6,       /* KV length update (prefill: done by the QKV GEMM) */
     VLA_STAGE_DEC_QKV = 7,      /* decode: RMSNorm + QKV + RoPE + KV append      */
     VLA_STAGE_DEC_ATTN = 8,     /* decode: split-KV attention + merge            */
     VLA_STAGE_DEC_O = 9,        /* decode: output projection + residual          */

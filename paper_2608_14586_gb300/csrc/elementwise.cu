@@ -7,28 +7,46 @@ namespace vla {
 
 namespace {
 
-// One thread per (row, 256-column chunk): fp32 sum of squares over the chunk's columns in
-// order, exactly as the residual GEMM epilogue accumulates its stored outputs.
+// Row sums of squares per 256-column chunk, in exactly the order the residual GEMM epilogue
+// forms them for its stored outputs: each 32-column group is an fp32 fmaf chain from zero over
+// its columns in order, and the chunk's sum adds the 8 group values in order. One thread per
+// group; the 8 threads of a chunk are consecutive lanes.
 __global__ void row_sumsq_kernel(const bf16* __restrict__ x, int M, int chunks, int ld, float* __restrict__ ss) {
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     pdl_wait();  // x is the previous kernel's output
     pdl_trigger();
-    if (i >= (long long)M * chunks) return;
-    const int row = (int)(i / chunks), t = (int)(i % chunks);
-    const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * ld + t * 256);
-    float acc = 0.f;
-#pragma unroll 4
-    for (int c = 0; c < 32; ++c) {
-        const uint4 v = xr[c];
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    const long long chunk = i >> 3;
+    const int grp = (int)(i & 7);
+    const bool ok = chunk < (long long)M * chunks;
+    float g = 0.f;
+    if (ok) {
+        const int row = (int)(chunk / chunks), t = (int)(chunk % chunks);
+        const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * ld + t * 256 + grp * 32);
+        uint4 v[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const float a = bf16_lo(w[k]), b = bf16_hi(w[k]);
-            acc = fmaf(a, a, acc);
-            acc = fmaf(b, b, acc);
+        for (int c = 0; c < 4; ++c) v[c] = xr[c];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint32_t w[4] = {v[c].x, v[c].y, v[c].z, v[c].w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float a = bf16_lo(w[k]), b = bf16_hi(w[k]);
+                g = fmaf(a, a, g);
+                g = fmaf(b, b, g);
+            }
         }
     }
-    ss[i] = acc;
+    // the chunk's 8 group sums to its first lane, added in group order
+    const int base = threadIdx.x & 24;  // first lane of this octet
+    float part[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) part[k] = __shfl_sync(0xFFFFFFFFu, g, base + k);
+    if (ok && grp == 0) {
+        float t = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t += part[k];
+        ss[chunk] = t;
+    }
 }
 
 // table[pos][j] = (cos, sin)(pos * base^(-2j/dh)), angles in float64
@@ -100,7 +118,7 @@ __global__ void set_lengths_kernel(int* d_len, int count, int value) {
 cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl) {
     if (M <= 0) return cudaSuccess;
     const int chunks = D / 256;
-    const long long n = (long long)M * chunks;
+    const long long n = (long long)M * chunks * 8;  // one thread per 32-column group
     return launch_ex(row_sumsq_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, stream, pdl, x, M, chunks, ld,
                      ss);
 }

@@ -63,14 +63,30 @@ VLA_DEV void store_bf16x32(bf16* dst, const float (&v)[32]) {
 VLA_DEV float row_rinv(const EpiParams& ep, int row) {
     const float* ps = ep.ss_in + (size_t)row * ep.ss_chunks;
     float t = 0.f;
-    for (int c = 0; c < ep.ss_chunks; ++c) t += ps[c];
+    if ((ep.ss_chunks & 3) == 0 && ep.ss_chunks <= 32) {  // 16-byte loads issued before the in-order sum
+        const int n4 = ep.ss_chunks >> 2;
+        float4 q[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) q[i] = i < n4 ? __ldcg(reinterpret_cast<const float4*>(ps) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            if (i < n4) {
+                t += q[i].x;
+                t += q[i].y;
+                t += q[i].z;
+                t += q[i].w;
+            }
+        }
+    } else {
+        for (int c = 0; c < ep.ss_chunks; ++c) t += ps[c];
+    }
     return 1.0f / sqrtf(t / (float)ep.norm_dim + ep.eps);
 }
 
 template <int BN>
 VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const bool row_ok = row < ep.M;
-    float ss = 0.f;  // sum of squares of the stored outputs, columns in order
+    float ss = 0.f;  // sum of squares of the stored outputs (32-column groups in order)
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
         uint32_t r[32];
@@ -98,12 +114,14 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
                 }
             }
             store_bf16x32(op, v);
-            if (ep.ss_out) {
+            if (ep.ss_out) {  // per 32 columns a chain from zero, the groups then added in order
+                float g = 0.f;
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const float r = __bfloat162float(__float2bfloat16_rn(v[i]));
-                    ss = fmaf(r, r, ss);
+                    g = fmaf(r, r, g);
                 }
+                ss += g;
             }
         } else {
 #pragma unroll
@@ -155,11 +173,14 @@ VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
             if (!row_ok) continue;
             float va[32], vb[32];
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const float2 cs = rope[c + i];
-                const float a = f32(ra[i]) * s, b = f32(rb[i]) * s;
-                va[i] = a * cs.x - b * cs.y;
-                vb[i] = b * cs.x + a * cs.y;
+            for (int i = 0; i < 32; i += 2) {  // 16-byte loads: two (cos, sin) pairs each
+                const float4 cs = __ldg(reinterpret_cast<const float4*>(rope + c + i));
+                const float a0 = f32(ra[i]) * s, b0 = f32(rb[i]) * s;
+                const float a1 = f32(ra[i + 1]) * s, b1 = f32(rb[i + 1]) * s;
+                va[i] = a0 * cs.x - b0 * cs.y;
+                vb[i] = b0 * cs.x + a0 * cs.y;
+                va[i + 1] = a1 * cs.z - b1 * cs.w;
+                vb[i + 1] = b1 * cs.z + a1 * cs.w;
             }
             if (region == 0) {
                 bf16* op = ep.out + (size_t)row * ep.ld_out + n0 + hb + c;
@@ -318,6 +339,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         pdl_wait();
         pdl_trigger();
+        // the layer's KV length advances with the keys this kernel writes (read only by later
+        // launches: decode takes the new token's position from it)
+        if (EPI == kEpiQKV && ep.len_out && blockIdx.x == 0 && lane == 0) *ep.len_out = ep.len_value;
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
             int stage = 0;

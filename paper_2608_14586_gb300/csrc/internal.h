@@ -40,6 +40,8 @@ struct EpiParams {
     bf16* vcache;
     const float2* rope;  // [max_ctx][head_dim/2] (cos, sin)
     int pos0, max_ctx, head_dim, q_cols, kv_cols;
+    int* len_out;   // kEpiQKV: the layer's device KV length, set to len_value (nullptr: leave)
+    int len_value;
     unsigned* status;
 };
 
@@ -83,9 +85,10 @@ cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status,
 // ---------------------------------------------------------------------------------------
 // Elementwise / setup kernels
 // ---------------------------------------------------------------------------------------
-// ss[i][t] = sum over columns [256t, 256t+256) of x[i][c]^2 (fp32, columns in order): the same
-// partial sums the residual GEMM epilogue writes for its output, so a block gets bit-identical
-// row statistics whether its input came from the previous block or from the caller.
+// ss[i][t] = sum over columns [256t, 256t+256) of x[i][c]^2 in fp32, formed as 8 in-order chains
+// over 32-column groups added in group order: the same partial sums the residual GEMM epilogue
+// writes for its output, so a block gets bit-identical row statistics whether its input came
+// from the previous block or from the caller.
 cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl = false);
 
 // cos/sin table [max_ctx][dh/2] from float64 angles pos * base^(-2j/dh)

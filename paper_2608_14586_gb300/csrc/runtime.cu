@@ -529,6 +529,8 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ep.head_dim = p->cfg.head_dim;
         ep.q_cols = p->qc;
         ep.kv_cols = p->kvc;
+        ep.len_out = kv->d_len + (l - kv->lb);
+        ep.len_value = p0 + M;
         ep.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_QKV, true);
         e = vla::launch_gemm(vla::kEpiQKV, qkv_bn, tm_x, qkv_bn == 128 ? ld.tm_qkv128 : ld.tm_qkv, M, p->qkv_n, D, ep,
@@ -604,12 +606,10 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         launches += 5;
     }
     if (e != cudaSuccess) return VLA_ERR_CUDA;
+    // device lengths were advanced by each layer's QKV kernel
     for (int l = layer_begin; l < layer_end; ++l) kv->len[l - kv->lb] = p0 + M;
-    stage_mark(p, VLA_STAGE_KV_LEN, true);
-    e = vla::launch_set_lengths(kv->d_len + (layer_begin - kv->lb), layer_end - layer_begin, p0 + M, stream);
-    stage_mark(p, VLA_STAGE_KV_LEN, false);
-    p->last_launches = launches + 1;
-    return cuda_status(e);
+    p->last_launches = launches;
+    return VLA_OK;
 }
 
 vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_begin, int layer_end, vla_kv* kv,
