@@ -377,6 +377,34 @@ def run_ours(args, dist: Dist):
         e2e = {"value": M * dist.world / (e2e_ms * 1e-3), "unit": "tokens/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": M * D * 2, "d2h_bytes_per_step": M * D * 2}
 
+    # ---- latency until one frame's boundary h^(16) is in host memory: the prefix followed by
+    # a device-to-host copy, vs the prefix whose last epilogue stores it to the host itself
+    boundary = None
+    if not args.no_e2e:
+        hb = torch.empty((M, D), dtype=torch.bfloat16).pin_memory()
+
+        def frame_to_host(fused: bool) -> float:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(main)
+            vla.vla_kv_reset(kv, main)
+            if fused:
+                vla.vla_prefix_prefill_to_host(p, x, M, 0, L, kv, outs[0], hb, main)
+            else:
+                vla.vla_prefix_prefill(p, x, M, 0, L, kv, outs[0], main)
+                vla.vla_boundary_to_host(outs[0], M, D, hb, main)
+            e1.record(main)
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1)
+
+        lat = {}
+        for fused in (False, True):
+            for _ in range(2):
+                frame_to_host(fused)
+            lat[fused] = statistics.median(frame_to_host(fused) for _ in range(max(5, args.steps // 3)))
+            assert torch.equal(hb.view(torch.int16), outs[0].view(torch.int16).cpu())
+        boundary = {"bytes": M * D * 2, "prefix_then_copy_ms": lat[False], "fused_store_ms": lat[True],
+                    "note": "one frame, from launch until h^(16) is in page-locked host memory (median)"}
+
     # ---- decode: 64 single-token steps against a 2304-position random context, in a cache
     # sized for the workload (2304 + 64 steps)
     decode = None
@@ -564,6 +592,7 @@ def run_ours(args, dist: Dist):
             "decode": decode,
             "pipeline": pipeline,
             "block_1024": block1k,
+            "boundary": boundary,
         }
         print(json.dumps(line), flush=True)
     vla.vla_kv_destroy(kv)

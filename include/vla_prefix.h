@@ -133,6 +133,18 @@ vla_status vla_kv_set_length(vla_kv* kv, int length, vla_stream stream);
 vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
                               vla_kv* kv, void* hidden_out, vla_stream stream);
 
+/* vla_prefix_prefill that also delivers h^(layer_end) to the host without a separate copy:
+ * the last block's down-projection epilogue stores each output tile both to hidden_out and,
+ * through the coherent CPU-GPU link, into page-locked host memory `pinned_dst` [n_tokens,
+ * hidden] bf16 (same layout). The boundary transfer T(.) of Eq. 6 then completes with the
+ * kernel: once an event recorded on `stream` after this call has completed, pinned_dst
+ * holds h^(layer_end). An empty range copies hidden_in to both. Errors: as prefill, plus
+ * NOT_PINNED (pinned_dst not page-locked or not mapped into the device address space) and
+ * INVALID_ARG (its device address not 16-byte aligned). */
+vla_status vla_prefix_prefill_to_host(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin,
+                                      int layer_end, vla_kv* kv, void* hidden_out, void* pinned_dst,
+                                      vla_stream stream);
+
 /* One autoregressive step of blocks [layer_begin, layer_end) on hidden_in [1, hidden] at
  * position = the range's common KV length; appends one K/V position per layer. Same
  * aliasing, range and error rules as prefill. */

@@ -18,7 +18,7 @@ __all__ = [
     "build", "load", "VlaError", "VlaConfig", "VlaLayerWeights",
     "vla_prefix_create", "vla_prefix_destroy", "vla_kv_create", "vla_kv_destroy", "vla_kv_reset",
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
-    "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
+    "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
     "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "STATUS", "STAGES",
 ]
@@ -83,6 +83,7 @@ def load():
         "vla_kv_set_length": ([P, I, V], I),
         "vla_prefix_prefill": ([P, V, I, I, I, P, V, V], I),
         "vla_prefix_decode": ([P, V, I, I, P, V, V], I),
+        "vla_prefix_prefill_to_host": ([P, V, I, I, I, P, V, V, V], I),
         "vla_boundary_to_host": ([V, I, I, V, V, V, V], I),
         "vla_last_async_error": ([P], I),
         "vla_status_str": ([I], ctypes.c_char_p),
@@ -203,6 +204,14 @@ def vla_prefix_prefill(p, hidden_in, n_tokens: int, layer_begin: int, layer_end:
                        stream=None):
     _check(load().vla_prefix_prefill(p, _ptr(hidden_in), n_tokens, layer_begin, layer_end, kv, _ptr(hidden_out),
                                      _stream(stream)), "vla_prefix_prefill")
+
+
+def vla_prefix_prefill_to_host(p, hidden_in, n_tokens: int, layer_begin: int, layer_end: int, kv, hidden_out,
+                               pinned_dst, stream=None):
+    """Prefill whose last block also stores h^(layer_end) into page-locked host memory."""
+    _check(load().vla_prefix_prefill_to_host(p, _ptr(hidden_in), n_tokens, layer_begin, layer_end, kv,
+                                             _ptr(hidden_out), _ptr(pinned_dst), _stream(stream)),
+           "vla_prefix_prefill_to_host")
 
 
 def vla_prefix_decode(p, hidden_in, layer_begin: int, layer_end: int, kv, hidden_out, stream=None):

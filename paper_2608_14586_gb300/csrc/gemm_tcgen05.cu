@@ -114,6 +114,7 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
                 }
             }
             store_bf16x32(op, v);
+            if (ep.out_host) store_bf16x32(ep.out_host + (size_t)row * ep.ld_out + col, v);
             if (ep.ss_out) {  // per 32 columns a chain from zero, the groups then added in order
                 float g = 0.f;
 #pragma unroll
@@ -130,6 +131,7 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
                     float x = v[i];
                     if (ep.resid) x += __bfloat162float(ep.resid[(size_t)row * ep.ld_resid + col + i]);
                     op[i] = __float2bfloat16_rn(x);
+                    if (ep.out_host) ep.out_host[(size_t)row * ep.ld_out + col + i] = op[i];
                 }
             }
         }

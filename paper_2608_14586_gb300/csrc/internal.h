@@ -24,6 +24,7 @@ struct EpiParams {
     int M, N;
     bf16* out;
     int ld_out;
+    bf16* out_host;  // kEpiResid: a second copy of the output rows (page-locked host memory, same layout)
     const bf16* resid;
     int ld_resid;
     // RMSNorm of the GEMM's input rows: 1/rms = 1/sqrt(sum_t ss_in[row][t] / D + eps), the

@@ -462,8 +462,10 @@ vla_status vla_kv_data(const vla_kv* kv, int layer, void** k_plane, void** v_pla
     return VLA_OK;
 }
 
-vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
-                              vla_kv* kv, void* hidden_out, vla_stream stream_) {
+// Prefill of [layer_begin, layer_end); with host_dev set, the last block's down projection
+// also stores h^(layer_end) into page-locked host memory (host_dev: its device address).
+static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
+                               vla_kv* kv, void* hidden_out, vla_stream stream_, bf16* host_dev, void* host_ptr) {
     if (!p || !hidden_in || !hidden_out || n_tokens < 0) return VLA_ERR_INVALID_ARG;
     if (!aligned16(hidden_in) || !aligned16(hidden_out)) return VLA_ERR_INVALID_ARG;
     if (n_tokens > p->cfg.max_ctx) return VLA_ERR_SHAPE;
@@ -475,8 +477,12 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
     cudaStream_t stream = (cudaStream_t)stream_;
     const int D = p->cfg.hidden, M = n_tokens;
     if (layer_begin == layer_end) {
-        if (hidden_in == hidden_out) return VLA_OK;
-        return cuda_status(cudaMemcpyAsync(hidden_out, hidden_in, (size_t)M * D * 2, cudaMemcpyDeviceToDevice, stream));
+        cudaError_t e = cudaSuccess;
+        if (hidden_in != hidden_out)
+            e = cudaMemcpyAsync(hidden_out, hidden_in, (size_t)M * D * 2, cudaMemcpyDeviceToDevice, stream);
+        if (e == cudaSuccess && host_ptr)
+            e = cudaMemcpyAsync(host_ptr, hidden_in, (size_t)M * D * 2, cudaMemcpyDeviceToHost, stream);
+        return cuda_status(e);
     }
     CUtensorMap tm_in, tm_out, tm_attn, tm_xmid, tm_m;
     if (!vla::make_tmap_bf16(&tm_in, hidden_in, M, D, D, 128) || !vla::make_tmap_bf16(&tm_out, hidden_out, M, D, D, 128) ||
@@ -597,6 +603,7 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
         ed.resid = p->ws_xmid;
         ed.ld_resid = D;
         ed.ss_out = (l + 1 < layer_end) ? p->ws_ss_x : nullptr;  // the next block's row statistics
+        ed.out_host = (l + 1 == layer_end) ? host_dev : nullptr;   // h^(layer_end) straight to the host
         ed.ss_chunks = D / 256;
         ed.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_DOWN, true);
@@ -610,6 +617,26 @@ vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens
     for (int l = layer_begin; l < layer_end; ++l) kv->len[l - kv->lb] = p0 + M;
     p->last_launches = launches;
     return VLA_OK;
+}
+
+vla_status vla_prefix_prefill(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
+                              vla_kv* kv, void* hidden_out, vla_stream stream) {
+    return prefill_impl(p, hidden_in, n_tokens, layer_begin, layer_end, kv, hidden_out, stream, nullptr, nullptr);
+}
+
+vla_status vla_prefix_prefill_to_host(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin,
+                                      int layer_end, vla_kv* kv, void* hidden_out, void* pinned_dst,
+                                      vla_stream stream) {
+    if (!pinned_dst) return VLA_ERR_INVALID_ARG;
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, pinned_dst) != cudaSuccess) {
+        cudaGetLastError();
+        return VLA_ERR_NOT_PINNED;
+    }
+    if (attr.type != cudaMemoryTypeHost || !attr.devicePointer) return VLA_ERR_NOT_PINNED;
+    if (!aligned16(attr.devicePointer)) return VLA_ERR_INVALID_ARG;
+    return prefill_impl(p, hidden_in, n_tokens, layer_begin, layer_end, kv, hidden_out, stream,
+                        static_cast<bf16*>(attr.devicePointer), pinned_dst);
 }
 
 vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_begin, int layer_end, vla_kv* kv,

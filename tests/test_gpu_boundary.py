@@ -147,3 +147,48 @@ def test_abi_errors_on_a_live_prefix(vla_lib):
     finally:
         m.close()
         other.close()
+
+
+@pytest.mark.parametrize("shape_name,L,M", [("TINY", 2, 64), ("B7", 2, 256)])
+def test_prefill_to_host_fused_boundary_store(vla_lib, shape_name, L, M):
+    """The last block's epilogue stores h^(L) into page-locked host memory as well: the host
+    copy, the device output and a plain prefill agree bit for bit; split ranges and the empty
+    range deliver the range's output; pageable memory is refused."""
+    import torch
+    vla = vla_lib
+    s = getattr(synth, shape_name)
+    m = Model(s, L, 5, M)
+    try:
+        x = to_dev(synth.hidden_states(M, s.hidden, 5))
+        kv = vla.vla_kv_create(m.handle, 0, L, M)
+        y_ref = torch.empty_like(x)
+        vla.vla_prefix_prefill(m.handle, x, M, 0, L, kv, y_ref)
+        host = torch.empty((M, s.hidden), dtype=torch.bfloat16, pin_memory=True)
+        host.view(torch.int16).fill_(-1)
+        y = torch.empty_like(x)
+        vla.vla_kv_reset(kv)
+        vla.vla_prefix_prefill_to_host(m.handle, x, M, 0, L, kv, y, host)
+        sync()
+        np.testing.assert_array_equal(_bits(y), _bits(y_ref))
+        np.testing.assert_array_equal(host.view(torch.int16).numpy(), _bits(y_ref))
+        # [0, 1) then [1, L) with the boundary of each range delivered to the host
+        h1 = torch.empty((M, s.hidden), dtype=torch.bfloat16, pin_memory=True)
+        mid = torch.empty_like(x)
+        vla.vla_kv_reset(kv)
+        vla.vla_prefix_prefill_to_host(m.handle, x, M, 0, 1, kv, mid, h1)
+        vla.vla_prefix_prefill_to_host(m.handle, mid, M, 1, L, kv, y, host)
+        sync()
+        np.testing.assert_array_equal(h1.view(torch.int16).numpy(), _bits(mid))
+        np.testing.assert_array_equal(host.view(torch.int16).numpy(), _bits(y_ref))
+        # empty range: the input itself
+        vla.vla_prefix_prefill_to_host(m.handle, x, M, 1, 1, None, y, host)
+        sync()
+        np.testing.assert_array_equal(host.view(torch.int16).numpy(), _bits(x))
+        pageable = np.zeros((M, s.hidden), dtype=np.uint16)
+        with pytest.raises(vla.VlaError) as ei:
+            vla.vla_prefix_prefill_to_host(m.handle, x, M, 0, L, kv, y, pageable.ctypes.data)
+        assert ei.value.name == "VLA_ERR_NOT_PINNED"
+        assert vla.vla_last_async_error(m.handle) == 0
+        vla.vla_kv_destroy(kv)
+    finally:
+        m.close()
