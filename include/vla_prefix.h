@@ -151,6 +151,15 @@ vla_status vla_prefix_prefill_to_host(vla_prefix* p, const void* hidden_in, int 
 vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_begin, int layer_end, vla_kv* kv,
                              void* hidden_out, vla_stream stream);
 
+/* One decode step for `batch` (1..4) independent sequences at once: hidden_in / hidden_out
+ * [batch, hidden] bf16 (row b = sequence b), kvs[b] = sequence b's cache (distinct caches of
+ * one max_ctx, each covering the range; each sequence at its own cache's common length).
+ * Every weight is streamed once for the whole batch. Each row equals what vla_prefix_decode
+ * returns for that sequence alone, bit for bit. Errors: as decode, plus SHAPE (batch out of
+ * range, caches of different max_ctx or first layer) and INVALID_ARG (a cache twice). */
+vla_status vla_prefix_decode_batch(vla_prefix* p, const void* hidden_in, int batch, int layer_begin, int layer_end,
+                                   vla_kv* const* kvs, void* hidden_out, vla_stream stream);
+
 /* The boundary transfer T(h^(p)) of Eq. 6: copies n_tokens x hidden bf16 (Eq. 11 bytes,
  * B = 1, b = 2) from device `hidden_out` into page-locked host memory `pinned_dst` on
  * `side_stream`, after `ready` (if non-NULL) and before recording `done` (if non-NULL), so

@@ -18,7 +18,7 @@ __all__ = [
     "build", "load", "VlaError", "VlaConfig", "VlaLayerWeights",
     "vla_prefix_create", "vla_prefix_destroy", "vla_kv_create", "vla_kv_destroy", "vla_kv_reset",
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
-    "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
+    "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_prefix_decode_batch", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
     "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "STATUS", "STAGES",
 ]
@@ -84,6 +84,7 @@ def load():
         "vla_prefix_prefill": ([P, V, I, I, I, P, V, V], I),
         "vla_prefix_decode": ([P, V, I, I, P, V, V], I),
         "vla_prefix_prefill_to_host": ([P, V, I, I, I, P, V, V, V], I),
+        "vla_prefix_decode_batch": ([P, V, I, I, I, ctypes.POINTER(P), V, V], I),
         "vla_boundary_to_host": ([V, I, I, V, V, V, V], I),
         "vla_last_async_error": ([P], I),
         "vla_status_str": ([I], ctypes.c_char_p),
@@ -217,6 +218,13 @@ def vla_prefix_prefill_to_host(p, hidden_in, n_tokens: int, layer_begin: int, la
 def vla_prefix_decode(p, hidden_in, layer_begin: int, layer_end: int, kv, hidden_out, stream=None):
     _check(load().vla_prefix_decode(p, _ptr(hidden_in), layer_begin, layer_end, kv, _ptr(hidden_out),
                                     _stream(stream)), "vla_prefix_decode")
+
+
+def vla_prefix_decode_batch(p, hidden_in, layer_begin: int, layer_end: int, kvs, hidden_out, stream=None):
+    """One decode step for len(kvs) sequences; hidden_in / hidden_out are [batch, hidden]."""
+    arr = (ctypes.c_void_p * len(kvs))(*[k.value if hasattr(k, "value") else k for k in kvs])
+    _check(load().vla_prefix_decode_batch(p, _ptr(hidden_in), len(kvs), layer_begin, layer_end, arr,
+                                          _ptr(hidden_out), _stream(stream)), "vla_prefix_decode_batch")
 
 
 def vla_boundary_to_host(hidden_out, n_tokens: int, hidden: int, pinned_dst, side_stream=None, ready=None,

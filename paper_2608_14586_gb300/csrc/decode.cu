@@ -18,6 +18,8 @@
 // predate the step before the wait, so the copy overlaps the QKV kernel), scores it for all
 // query heads of the GQA group with an online softmax, and the cluster merges the partial
 // (max, sum, output) states through distributed shared memory in fixed rank order.
+#include <cstring>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -27,17 +29,20 @@ namespace {
 
 enum GemvMode : int { kGemvQKV = 0, kGemvResid = 1, kGemvSwiGLU = 2 };
 
+// A batch of NB token vectors (NB <= kMaxDecodeBatch), each of its own sequence: the
+// weights stream once for all of them. Per-sequence arrays are [NB][...] with the stride of
+// one vector.
 struct GemvParams {
     const bf16* W;  // [rows, K] row-major
     int K;          // multiple of 256
     int units;      // row pairs
-    const bf16* xv;     // input vector [K]
-    const bf16* resid;  // kGemvResid: residual [2*units]
-    bf16* out;          // kGemvResid: [2*units]; kGemvSwiGLU: [units]
-    float* q_out;       // kGemvQKV: post-RoPE query, fp32 [H*dh]
-    bf16* kcache;
-    bf16* vcache;
-    const int* d_len;  // kGemvQKV: position of the new token
+    const bf16* xv;     // input vectors [NB][K]
+    const bf16* resid;  // kGemvResid: residual [NB][2*units]
+    bf16* out;          // kGemvResid: [NB][2*units]; kGemvSwiGLU: [NB][units]
+    float* q_out;       // kGemvQKV: post-RoPE queries, fp32 [NB][H*dh]
+    bf16* kcache[kMaxDecodeBatch];  // kGemvQKV: each sequence's layer K / V planes
+    bf16* vcache[kMaxDecodeBatch];
+    const int* d_len[kMaxDecodeBatch];  // kGemvQKV: position of each sequence's new token
     const float2* rope;
     int dh, n_q_heads, n_kv_heads, max_ctx;
     float eps;
@@ -75,47 +80,50 @@ VLA_DEV void unit_rows(const GemvParams& p, int u, int& ra, int& rb) {
     }
 }
 
-// Fused epilogue of one row pair (lane 0 of the warp that reduced it).
+// Fused epilogue of one row pair for sequence b (lane 0 of the warp that reduced it).
 template <int MODE>
-VLA_DEV void gemv_epilogue(const GemvParams& p, int u, int ra, int rb, float acc_a, float acc_b, float rinv, int pos) {
+VLA_DEV void gemv_epilogue(const GemvParams& p, int b, int u, int ra, int rb, float acc_a, float acc_b, float rinv,
+                           int pos) {
     if constexpr (MODE == kGemvResid) {
-        const float ya = __bfloat162float(p.resid[ra]) + acc_a;
-        const float yb = __bfloat162float(p.resid[rb]) + acc_b;
-        *reinterpret_cast<uint32_t*>(p.out + ra) = pack_bf16x2(ya, yb);
+        const size_t n = (size_t)2 * p.units * b;
+        const float ya = __bfloat162float(p.resid[n + ra]) + acc_a;
+        const float yb = __bfloat162float(p.resid[n + rb]) + acc_b;
+        *reinterpret_cast<uint32_t*>(p.out + n + ra) = pack_bf16x2(ya, yb);
     } else if constexpr (MODE == kGemvSwiGLU) {
         const float g = acc_a * rinv, up = acc_b * rinv;
-        p.out[u] = __float2bfloat16_rn(g / (1.0f + __expf(-g)) * up);
+        p.out[(size_t)p.units * b + u] = __float2bfloat16_rn(g / (1.0f + __expf(-g)) * up);
     } else {
         const int half = p.dh >> 1;
         const int head = u / half, j = u % half;
-        float a = acc_a * rinv, b = acc_b * rinv;
+        float a = acc_a * rinv, bb = acc_b * rinv;
         if (head < p.n_q_heads + p.n_kv_heads) {
             const float2 cs = p.rope[(size_t)pos * half + j];
-            const float a2 = a * cs.x - b * cs.y;
-            const float b2 = b * cs.x + a * cs.y;
+            const float a2 = a * cs.x - bb * cs.y;
+            const float b2 = bb * cs.x + a * cs.y;
             a = a2;
-            b = b2;
+            bb = b2;
         }
         if (head < p.n_q_heads) {
-            p.q_out[head * p.dh + j] = a;
-            p.q_out[head * p.dh + j + half] = b;
+            float* q = p.q_out + (size_t)b * p.n_q_heads * p.dh;
+            q[head * p.dh + j] = a;
+            q[head * p.dh + j + half] = bb;
         } else if (head < p.n_q_heads + p.n_kv_heads) {
-            bf16* kp = p.kcache + ((size_t)(head - p.n_q_heads) * p.max_ctx + pos) * p.dh;
+            bf16* kp = p.kcache[b] + ((size_t)(head - p.n_q_heads) * p.max_ctx + pos) * p.dh;
             kp[j] = __float2bfloat16_rn(a);
-            kp[j + half] = __float2bfloat16_rn(b);
+            kp[j + half] = __float2bfloat16_rn(bb);
         } else {
-            bf16* vp = p.vcache + ((size_t)(head - p.n_q_heads - p.n_kv_heads) * p.max_ctx + pos) * p.dh;
+            bf16* vp = p.vcache[b] + ((size_t)(head - p.n_q_heads - p.n_kv_heads) * p.max_ctx + pos) * p.dh;
             vp[j] = __float2bfloat16_rn(a);
-            vp[j + half] = __float2bfloat16_rn(b);
+            vp[j + half] = __float2bfloat16_rn(bb);
         }
     }
 }
 
-template <int MODE>
-__global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
-    extern __shared__ uint4 xs[];
-    __shared__ float red[kGemvThreads / 32];
-    __shared__ float s_rinv;
+template <int MODE, int NB>
+__global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_constant__ GemvParams p) {
+    extern __shared__ uint4 xs[];  // [NB][K/8]
+    __shared__ float red[NB][kGemvThreads / 32];
+    __shared__ float s_rinv[NB];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int gw = blockIdx.x * (kGemvThreads / 32) + warp;
     const int nw = gridDim.x * (kGemvThreads / 32);
@@ -149,36 +157,49 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
     pdl_wait();
     pdl_trigger();
     const uint4* xg = reinterpret_cast<const uint4*>(p.xv);
-    for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) xs[i] = __ldcg(xg + i);
+    for (int i = threadIdx.x; i < NB * nchunk; i += kGemvThreads) xs[i] = __ldcg(xg + i);
     __syncthreads();
-    float rinv = 1.f;
+    float rinv[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) rinv[b] = 1.f;
     if constexpr (MODE != kGemvResid) {
-        float ss = 0.f;
-        for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) {
-            const uint4 v = xs[i];
-            ss += dot8(v, v);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            float ss = 0.f;
+            for (int i = threadIdx.x; i < nchunk; i += kGemvThreads) {
+                const uint4 v = xs[b * nchunk + i];
+                ss += dot8(v, v);
+            }
+            ss = warp_sum(ss);
+            if (lane == 0) red[b][warp] = ss;
         }
-        ss = warp_sum(ss);
-        if (lane == 0) red[warp] = ss;
         __syncthreads();
-        if (threadIdx.x == 0) {
+        if (threadIdx.x < NB) {
             float t = 0.f;
-            for (int w = 0; w < kGemvThreads / 32; ++w) t += red[w];
-            s_rinv = 1.0f / sqrtf(t / (float)p.K + p.eps);
+            for (int w = 0; w < kGemvThreads / 32; ++w) t += red[threadIdx.x][w];
+            s_rinv[threadIdx.x] = 1.0f / sqrtf(t / (float)p.K + p.eps);
         }
         __syncthreads();
-        rinv = s_rinv;
+#pragma unroll
+        for (int b = 0; b < NB; ++b) rinv[b] = s_rinv[b];
     }
 
-    int pos = 0;
-    if constexpr (MODE == kGemvQKV) pos = *p.d_len;
+    int pos[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) pos[b] = 0;
+    if constexpr (MODE == kGemvQKV) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b) pos[b] = *p.d_len[b];
+    }
 
     for (int u = gw; u < p.units; u += nw) {
         int ra, rb;
         unit_rows<MODE>(p, u, ra, rb);
         const uint4* wa = reinterpret_cast<const uint4*>(p.W + (size_t)ra * p.K);
         const uint4* wb = reinterpret_cast<const uint4*>(p.W + (size_t)rb * p.K);
-        float acc_a = 0.f, acc_b = 0.f;
+        float acc_a[NB], acc_b[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) acc_a[b] = acc_b[b] = 0.f;
         for (int s = 0; s < nstep; s += kGemvU) {
 #pragma unroll
             for (int i = 0; i < kGemvU; ++i) {
@@ -191,15 +212,21 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
 #pragma unroll
             for (int i = 0; i < kGemvU; ++i) {
                 if (s + i < nstep) {
-                    const uint4 x = xs[(s + i) * 32 + lane];
-                    acc_a += dot8(va[i], x);
-                    acc_b += dot8(vb[i], x);
+#pragma unroll
+                    for (int b = 0; b < NB; ++b) {
+                        const uint4 x = xs[b * nchunk + (s + i) * 32 + lane];
+                        acc_a[b] += dot8(va[i], x);
+                        acc_b[b] += dot8(vb[i], x);
+                    }
                 }
             }
         }
-        acc_a = warp_sum(acc_a);
-        acc_b = warp_sum(acc_b);
-        if (lane == 0) gemv_epilogue<MODE>(p, u, ra, rb, acc_a, acc_b, rinv, pos);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const float sa = warp_sum(acc_a[b]);
+            const float sb = warp_sum(acc_b[b]);
+            if (lane == 0) gemv_epilogue<MODE>(p, b, u, ra, rb, sa, sb, rinv[b], pos[b]);
+        }
     }
 }
 
@@ -207,16 +234,16 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(GemvParams p) {
 // split-KV attention: one thread-block cluster per KV head
 // ---------------------------------------------------------------------------------------
 struct AttnDecParams {
-    const float* q;  // [H*dh] post-RoPE query, fp32
-    const bf16* kc;  // layer base [Hkv][max_ctx][dh]
-    const bf16* vc;
-    const int* d_len;  // position of the new token; context = d_len + 1
-    int H, Hkv, max_ctx;
+    const float* q;  // [nb][H*dh] post-RoPE queries, fp32
+    const bf16* kc[kMaxDecodeBatch];  // each sequence's layer base [Hkv][max_ctx][dh]
+    const bf16* vc[kMaxDecodeBatch];
+    const int* d_len[kMaxDecodeBatch];  // positions of the new tokens; context = d_len + 1
+    int nb, H, Hkv, max_ctx;
     int cs;      // CTAs per cluster = key splits per KV head
     int cap;     // keys per shared-memory stage
     int stages;  // 1 or 2
     float scale_log2;
-    bf16* out;  // [H*dh] attention output
+    bf16* out;  // [nb][H*dh] attention outputs
     unsigned* status;
 };
 
@@ -244,7 +271,7 @@ VLA_DEV void load_row_part(const bf16* src, float (&f)[DPL]) {
 // r merges output elements [r*G*dh/cs, (r+1)*G*dh/cs) over the cs CTAs through distributed
 // shared memory, in fixed rank order, and writes them. No partials leave the chip.
 template <int DH, int G>
-__global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams p) {
+__global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(const __grid_constant__ AttnDecParams p) {
     constexpr int DPL = DH / 16;
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ uint64_t full[2];
@@ -253,13 +280,15 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
     __shared__ float c_m[G], c_l[G];
     __shared__ __align__(16) float c_o[G * DH];
     __shared__ int s_ok;
-    const int rank = blockIdx.x, kvh = blockIdx.y;
+    const int rank = blockIdx.x, kvh = blockIdx.y, seq = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bf16* kc = p.kc[seq];
+    const bf16* vc = p.vc[seq];
     const int sub = lane >> 4, l16 = lane & 15;
     const size_t stage_elems = (size_t)2 * p.cap * DH;  // K rows then V rows
     bf16* const sbase = reinterpret_cast<bf16*>(smem);
     // d_len was last written by an earlier step (complete before this one started)
-    const int ctx = *p.d_len + 1;
+    const int ctx = *p.d_len[seq] + 1;
     const int per = (ctx + p.cs - 1) / p.cs;
     const int kb = rank * per;
     const int ke = min(ctx, kb + per);
@@ -277,8 +306,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
         mbar_arrive_expect_tx(bar, 2u * bytes);
         if (bytes) {
             const size_t off = ((size_t)kvh * p.max_ctx + r0) * DH;
-            bulk_load(sk, p.kc + off, bytes, bar);
-            bulk_load(sk + (size_t)p.cap * DH, p.vc + off, bytes, bar);
+            bulk_load(sk, kc + off, bytes, bar);
+            bulk_load(sk + (size_t)p.cap * DH, vc + off, bytes, bar);
         }
     };
     if (tid == 0) {
@@ -294,7 +323,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
 #pragma unroll
     for (int hh = 0; hh < G; ++hh)
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) qv[hh][d] = __ldcg(p.q + (kvh * G + hh) * DH + l16 * DPL + d) * p.scale_log2;
+        for (int d = 0; d < DPL; ++d)
+            qv[hh][d] = __ldcg(p.q + ((size_t)seq * p.H + kvh * G + hh) * DH + l16 * DPL + d) * p.scale_log2;
     float m[G], l[G], o[G][DPL];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
@@ -313,9 +343,9 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
         if (nr >= 0 && nr < rows && tid < DH / 8) {
             const size_t off = ((size_t)kvh * p.max_ctx + new_row) * DH;
             reinterpret_cast<uint4*>(const_cast<bf16*>(sk) + (size_t)nr * DH)[tid] =
-                __ldcg(reinterpret_cast<const uint4*>(p.kc + off) + tid);
+                __ldcg(reinterpret_cast<const uint4*>(kc + off) + tid);
             reinterpret_cast<uint4*>(const_cast<bf16*>(sv) + (size_t)nr * DH)[tid] =
-                __ldcg(reinterpret_cast<const uint4*>(p.vc + off) + tid);
+                __ldcg(reinterpret_cast<const uint4*>(vc + off) + tid);
         }
         if (!mbar_wait(&full[c % p.stages], (uint32_t)(c / p.stages) & 1u)) s_ok = 0;
         __syncthreads();
@@ -425,30 +455,47 @@ __global__ void __launch_bounds__(kAttnThreads) attn_decode_kernel(AttnDecParams
                 ot = fmaf(orr[r], cw, ot);
             }
         }
-        p.out[kvh * G * DH + e] = __float2bfloat16_rn(ot / lt);
+        p.out[((size_t)seq * p.H + kvh * G) * DH + e] = __float2bfloat16_rn(ot / lt);
     }
     cluster_sync_all();  // keep this CTA's shared memory alive until the cluster has read it
 }
 
-__global__ void advance_lengths_kernel(int* d_len, int count) {
+struct LenPtrs {
+    int* p[kMaxDecodeBatch];
+};
+
+// block b: the sequence's layer lengths += 1
+__global__ void advance_lengths_kernel(const __grid_constant__ LenPtrs lp, int count) {
     const int i = threadIdx.x;
-    if (i < count) d_len[i] += 1;
+    if (i < count) lp.p[blockIdx.x][i] += 1;
 }
 
-template <int MODE>
-cudaError_t launch_gemv(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
-    const size_t smem = (size_t)p.K * 2;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+template <int MODE, int NB>
+cudaError_t launch_gemv_nb(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
+    const size_t smem = (size_t)NB * p.K * 2;
+    static size_t attr = 0;
+    if (smem > attr) {
+        cudaError_t e =
+            cudaFuncSetAttribute(gemv_kernel<MODE, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr = smem;
     }
     const int warps_needed = p.units;
     int grid = 2 * num_sms;
     const int gmax = (warps_needed + 7) / 8;
     if (grid > gmax) grid = gmax;
-    return launch_ex(gemv_kernel<MODE>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
+    return launch_ex(gemv_kernel<MODE, NB>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
+}
+
+template <int MODE>
+cudaError_t launch_gemv(const GemvParams& p, int nb, int num_sms, cudaStream_t s, bool pdl) {
+    switch (nb) {
+        case 1: return launch_gemv_nb<MODE, 1>(p, num_sms, s, pdl);
+        case 2: return launch_gemv_nb<MODE, 2>(p, num_sms, s, pdl);
+        case 3: return launch_gemv_nb<MODE, 3>(p, num_sms, s, pdl);
+        case 4: return launch_gemv_nb<MODE, 4>(p, num_sms, s, pdl);
+    }
+    return cudaErrorInvalidValue;
 }
 
 template <int DH, int G>
@@ -477,7 +524,7 @@ cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s, bool pdl) {
         attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.cs, p.Hkv);
+    cfg.gridDim = dim3(p.cs, p.Hkv, p.nb);
     cfg.blockDim = dim3(kAttnThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
@@ -573,6 +620,7 @@ cudaError_t plan_decode_attention(int dh, int group, int Hkv, int max_ctx, int* 
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
                                 bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook, bool pdl_first) {
     cudaError_t e;
+    if (L.nb < 1 || L.nb > kMaxDecodeBatch) return cudaErrorInvalidValue;
     // stage timing records events between the launches: launch those fully serialized
     const bool pdl = hook.fn == nullptr && pdl_enabled();
     pdl_first = pdl_first && pdl;
@@ -584,9 +632,11 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     g.units = (qc + 2 * kvc) / 2;
     g.xv = x_in;
     g.q_out = w.q;
-    g.kcache = L.kcache;
-    g.vcache = L.vcache;
-    g.d_len = L.d_len;
+    for (int b = 0; b < L.nb; ++b) {
+        g.kcache[b] = L.kcache[b];
+        g.vcache[b] = L.vcache[b];
+        g.d_len[b] = L.d_len[b];
+    }
     g.rope = w.rope;
     g.dh = d.dh;
     g.n_q_heads = d.H;
@@ -594,45 +644,53 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     g.max_ctx = d.max_ctx;
     g.eps = d.eps;
     hook(kStageDecQKV, true);
-    e = launch_gemv<kGemvQKV>(g, num_sms, stream, pdl_first);
+    e = launch_gemv<kGemvQKV>(g, L.nb, num_sms, stream, pdl_first);
     hook(kStageDecQKV, false);
     if (e != cudaSuccess) return e;
-    // 2. split-KV attention + combine
-    AttnDecParams a = {};
-    a.q = w.q;
-    a.kc = L.kcache;
-    a.vc = L.vcache;
-    a.d_len = L.d_len;
-    a.H = d.H;
-    a.Hkv = d.Hkv;
-    a.max_ctx = d.max_ctx;
-    a.cs = w.attn_cs;
-    a.cap = w.attn_cap;
-    a.stages = w.attn_stages;
-    a.scale_log2 = 1.4426950408889634f / sqrtf((float)d.dh);
-    a.out = w.attn;
-    a.status = w.status;
+    // 2. split-KV attention, one cluster per (sequence, KV head)
+    const float scale_log2 = 1.4426950408889634f / sqrtf((float)d.dh);
     hook(kStageDecAttn, true);
     if (w.attn_tc) {
-        CUtensorMap tk, tv;
-        if (!make_tmap_bf16_3d(&tk, L.kcache, d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32) ||
-            !make_tmap_bf16_3d(&tv, L.vcache, d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32))
-            return cudaErrorInvalidValue;
+        DecKVMaps maps;
+        memset(&maps, 0, sizeof(maps));
         AttnDecTcParams t = {};
+        for (int b = 0; b < L.nb; ++b) {
+            if (!make_tmap_bf16_3d(&maps.k[b], L.kcache[b], d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32) ||
+                !make_tmap_bf16_3d(&maps.v[b], L.vcache[b], d.dh, d.max_ctx, d.Hkv, (uint64_t)d.max_ctx * d.dh, 32))
+                return cudaErrorInvalidValue;
+            t.kc[b] = L.kcache[b];
+            t.vc[b] = L.vcache[b];
+            t.d_len[b] = L.d_len[b];
+        }
         t.q = w.q;
-        t.kc = L.kcache;
-        t.vc = L.vcache;
-        t.d_len = L.d_len;
+        t.nb = L.nb;
         t.H = d.H;
         t.Hkv = d.Hkv;
         t.max_ctx = d.max_ctx;
         t.cs = w.attn_cs;
         t.rows = w.attn_cap;
-        t.scale_log2 = a.scale_log2;
+        t.scale_log2 = scale_log2;
         t.out = w.attn;
         t.status = w.status;
-        e = launch_attn_decode_tc(tk, tv, d.H / d.Hkv, t, stream, pdl);
+        e = launch_attn_decode_tc(maps, d.H / d.Hkv, t, stream, pdl);
     } else {
+        AttnDecParams a = {};
+        for (int b = 0; b < L.nb; ++b) {
+            a.kc[b] = L.kcache[b];
+            a.vc[b] = L.vcache[b];
+            a.d_len[b] = L.d_len[b];
+        }
+        a.q = w.q;
+        a.nb = L.nb;
+        a.H = d.H;
+        a.Hkv = d.Hkv;
+        a.max_ctx = d.max_ctx;
+        a.cs = w.attn_cs;
+        a.cap = w.attn_cap;
+        a.stages = w.attn_stages;
+        a.scale_log2 = scale_log2;
+        a.out = w.attn;
+        a.status = w.status;
         e = launch_attn_dec_any(d.dh, d.H / d.Hkv, a, stream, pdl);
     }
     hook(kStageDecAttn, false);
@@ -646,7 +704,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     o.resid = x_in;
     o.out = w.x_mid;
     hook(kStageDecO, true);
-    e = launch_gemv<kGemvResid>(o, num_sms, stream, pdl);
+    e = launch_gemv<kGemvResid>(o, L.nb, num_sms, stream, pdl);
     hook(kStageDecO, false);
     if (e != cudaSuccess) return e;
     // 4. RMSNorm + gate/up + SwiGLU
@@ -658,7 +716,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     gu.out = w.m;
     gu.eps = d.eps;
     hook(kStageDecGateUp, true);
-    e = launch_gemv<kGemvSwiGLU>(gu, num_sms, stream, pdl);
+    e = launch_gemv<kGemvSwiGLU>(gu, L.nb, num_sms, stream, pdl);
     hook(kStageDecGateUp, false);
     if (e != cudaSuccess) return e;
     // 5. down projection + residual
@@ -670,14 +728,17 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     dn.resid = w.x_mid;
     dn.out = x_out;
     hook(kStageDecDown, true);
-    e = launch_gemv<kGemvResid>(dn, num_sms, stream, pdl);
+    e = launch_gemv<kGemvResid>(dn, L.nb, num_sms, stream, pdl);
     hook(kStageDecDown, false);
     return e;
 }
 
-cudaError_t launch_advance_lengths(int* d_len, int count, cudaStream_t stream) {
-    if (count <= 0) return cudaSuccess;
-    advance_lengths_kernel<<<1, ((count + 31) / 32) * 32, 0, stream>>>(d_len, count);
+cudaError_t launch_advance_lengths(int* const* d_len, int nb, int count, cudaStream_t stream) {
+    if (count <= 0 || nb <= 0) return cudaSuccess;
+    if (nb > kMaxDecodeBatch) return cudaErrorInvalidValue;
+    LenPtrs lp = {};
+    for (int b = 0; b < nb; ++b) lp.p[b] = d_len[b];
+    advance_lengths_kernel<<<nb, ((count + 31) / 32) * 32, 0, stream>>>(lp, count);
     return cudaGetLastError();
 }
 

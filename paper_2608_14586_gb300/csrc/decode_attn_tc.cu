@@ -1,6 +1,6 @@
 // Single-token (decode) attention on the 5th-generation tensor cores, head_dim 128.
 //
-// One thread-block cluster of `cs` CTAs per KV head g; CTA rank r owns the contiguous key range
+// One thread-block cluster of `cs` CTAs per (sequence, KV head g); CTA rank r owns the contiguous key range
 // [r*ceil(ctx/cs), ...) of the context (Sec. 3.2's causal attention at one query position,
 // split over keys). Per CTA, for the G query heads of the GQA group:
 //   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory
@@ -65,8 +65,7 @@ __host__ __device__ inline uint32_t half_off(int rows, int t, int half) {
 
 template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_decode_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                          AttnDecTcParams p) {
+    attn_decode_tc_kernel(const __grid_constant__ DecKVMaps maps, const __grid_constant__ AttnDecTcParams p) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint64_t bar_kv, bar_mma;
     __shared__ uint32_t tmem_slot;
@@ -81,11 +80,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* sV = smem + L.off_v;
     uint8_t* sQ = smem + L.off_q;
     uint8_t* sP = smem + L.off_p;
-    const int rank = blockIdx.x, kvh = blockIdx.y;
+    const int rank = blockIdx.x, kvh = blockIdx.y, seq = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const CUtensorMap* tmK = &maps.k[seq];
+    const CUtensorMap* tmV = &maps.v[seq];
+    const bf16* kc = p.kc[seq];
+    const bf16* vc = p.vc[seq];
+    const float* q = p.q + (size_t)seq * p.H * kDH;
 
     // d_len was last written by an earlier step (complete before this one started)
-    const int ctx = *p.d_len + 1;
+    const int ctx = *p.d_len[seq] + 1;
     const int per = (ctx + p.cs - 1) / p.cs;
     const int kb = rank * per;
     const int nk = max(0, min(min(ctx, kb + per) - kb, p.rows));
@@ -97,8 +101,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&bar_mma, 1);
         fence_barrier_init();
         s_ok = 1;
-        tma_prefetch_desc(&tmK);
-        tma_prefetch_desc(&tmV);
+        tma_prefetch_desc(tmK);
+        tma_prefetch_desc(tmV);
     }
     if (warp == 0) {
         tmem_alloc(&tmem_slot, kTmemCols);
@@ -117,8 +121,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int y = kb + b * kBoxRows;
             for (int c = 0; c < 2; ++c) {
                 const uint32_t dst = half_off(p.rows, b >> 2, c) + (uint32_t)(b & 3) * kBoxBytes;
-                tma_load_3d(sK + dst, &tmK, &bar_kv, c * 64, y, kvh);
-                tma_load_3d(sV + dst, &tmV, &bar_kv, c * 64, y, kvh);
+                tma_load_3d(sK + dst, tmK, &bar_kv, c * 64, y, kvh);
+                tma_load_3d(sV + dst, tmV, &bar_kv, c * 64, y, kvh);
             }
         }
     }
@@ -128,7 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Q (post-RoPE, fp32) -> bf16 rows [0, G) of the swizzled K-major tile
     for (int i = tid; i < G * 16; i += kThreads) {
         const int hh = i >> 4, j = i & 15;  // head, 16-byte chunk of 8 dims
-        const float4* src = reinterpret_cast<const float4*>(p.q + (size_t)(kvh * G + hh) * kDH + j * 8);
+        const float4* src = reinterpret_cast<const float4*>(q + (size_t)(kvh * G + hh) * kDH + j * 8);
         const float4 a = __ldcg(src), b = __ldcg(src + 1);
         *reinterpret_cast<uint4*>(sQ + (j >> 3) * (16 * 128) + sw128_off(hh, j & 7)) =
             make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
@@ -138,7 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // zero probabilities never meet non-finite values
     if (new_row >= 0 && new_row < nk && tid < 32) {
         const int half = tid >> 4, j = (tid >> 1) & 7, which = tid & 1;  // 2 halves x 8 chunks x {K, V}
-        const bf16* src = (which ? p.vc : p.kc) + ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + half * 64 + j * 8;
+        const bf16* src = (which ? vc : kc) + ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + half * 64 + j * 8;
         uint8_t* dst = (which ? sV : sK) + half_off(p.rows, new_row >> 7, half) + sw128_off(new_row & 127, j);
         *reinterpret_cast<uint4*>(dst) = __ldcg(reinterpret_cast<const uint4*>(src));
     }
@@ -301,7 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ot = fmaf(orr[r], cw, ot);
             }
         }
-        p.out[(size_t)kvh * G * kDH + e] = __float2bfloat16_rn(ot / lt);
+        p.out[((size_t)seq * p.H + kvh * G) * kDH + e] = __float2bfloat16_rn(ot / lt);
     }
     cluster_sync_all();  // keep this CTA's shared memory alive until the cluster has read it
 }
@@ -316,7 +320,7 @@ cudaError_t prepare(int cs, size_t smem) {
 }
 
 template <int G>
-cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTcParams& p, cudaStream_t s, bool pdl) {
+cudaError_t launch(const DecKVMaps& maps, const AttnDecTcParams& p, cudaStream_t s, bool pdl) {
     const size_t smem = smem_layout(p.rows).total;
     static size_t attr_smem = 0;
     static int attr_cs = 0;
@@ -327,7 +331,7 @@ cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTc
         attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.cs, p.Hkv);
+    cfg.gridDim = dim3(p.cs, p.Hkv, p.nb);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
@@ -340,7 +344,7 @@ cudaError_t launch(const CUtensorMap& tk, const CUtensorMap& tv, const AttnDecTc
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 2 : 1;
-    return cudaLaunchKernelEx(&cfg, attn_decode_tc_kernel<G>, tk, tv, p);
+    return cudaLaunchKernelEx(&cfg, attn_decode_tc_kernel<G>, maps, p);
 }
 
 // Cluster size 16 (else 8) with each CTA holding ceil(max_ctx / cs) keys; preferred when all
@@ -399,13 +403,13 @@ bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, 
     return false;
 }
 
-cudaError_t launch_attn_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, int group, const AttnDecTcParams& p,
-                                  cudaStream_t s, bool pdl) {
+cudaError_t launch_attn_decode_tc(const DecKVMaps& maps, int group, const AttnDecTcParams& p, cudaStream_t s,
+                                  bool pdl) {
     switch (group) {
-        case 1: return launch<1>(tk, tv, p, s, pdl);
-        case 2: return launch<2>(tk, tv, p, s, pdl);
-        case 4: return launch<4>(tk, tv, p, s, pdl);
-        case 8: return launch<8>(tk, tv, p, s, pdl);
+        case 1: return launch<1>(maps, p, s, pdl);
+        case 2: return launch<2>(maps, p, s, pdl);
+        case 4: return launch<4>(maps, p, s, pdl);
+        case 8: return launch<8>(maps, p, s, pdl);
     }
     return cudaErrorInvalidValue;
 }

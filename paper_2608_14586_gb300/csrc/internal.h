@@ -111,44 +111,53 @@ cudaError_t launch_repack(const RepackSrc& s, const RepackDst& d, int D, int H, 
 cudaError_t launch_set_lengths(int* d_len, int count, int value, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------------------
-// Decode (one token): weight-streaming GEMVs and split-KV attention
+// Decode (one token per sequence, up to kMaxDecodeBatch sequences): weight-streaming GEMVs
+// and split-KV attention
 // ---------------------------------------------------------------------------------------
+constexpr int kMaxDecodeBatch = 4;
+// One block of a decode step for nb sequences (one token each, each with its own KV cache).
 struct DecodeLayer {
     const bf16 *w_qkv, *w_o, *w_gu, *w_d;
-    bf16* kcache;  // layer base [Hkv][max_ctx][dh]
-    bf16* vcache;
-    const int* d_len;  // this layer's device length (position of the new token)
+    int nb;
+    bf16* kcache[kMaxDecodeBatch];  // each sequence's layer base [Hkv][max_ctx][dh]
+    bf16* vcache[kMaxDecodeBatch];
+    const int* d_len[kMaxDecodeBatch];  // each sequence's device length for this layer (new position)
 };
 struct DecodeDims {
     int D, H, Hkv, dh, F_pad, max_ctx;
     float eps;
 };
 struct DecodeWork {
-    float* q;          // [H*dh] fp32 (post-RoPE query)
-    bf16* attn;        // [H*dh]
-    bf16* x_mid;       // [D]
-    bf16* m;           // [F_pad]
+    float* q;          // [nb][H*dh] fp32 (post-RoPE queries)
+    bf16* attn;        // [nb][H*dh]
+    bf16* x_mid;       // [nb][D]
+    bf16* m;           // [nb][F_pad]
     const float2* rope;
     unsigned* status;
     int attn_tc;                         // 1: tcgen05 kernel (attn_cap = keys per CTA), 0: CUDA-core kernel
     int attn_cs, attn_cap, attn_stages;  // from plan_decode_attention(_tc)
 };
-// Decode attention on tcgen05 (head_dim 128): one cluster of `cs` CTAs per KV head, each
-// holding up to `rows` keys (a multiple of 32, at most 384). K/V tensor maps: 3-D [Hkv][max_ctx][128] bf16 maps of the
-// layer's cache planes with 32-row boxes (make_tmap_bf16_3d).
+// Decode attention on tcgen05 (head_dim 128): one cluster of `cs` CTAs per (sequence, KV
+// head), each CTA holding up to `rows` keys (a multiple of 32, at most 384). K/V tensor maps:
+// 3-D [Hkv][max_ctx][128] bf16 maps of each sequence's layer planes with 32-row boxes
+// (make_tmap_bf16_3d).
+struct DecKVMaps {
+    CUtensorMap k[kMaxDecodeBatch];
+    CUtensorMap v[kMaxDecodeBatch];
+};
 struct AttnDecTcParams {
-    const float* q;     // [H*dh] post-RoPE query, fp32
-    const bf16* kc;     // layer base [Hkv][max_ctx][dh] (the new token's row is read directly)
-    const bf16* vc;
-    const int* d_len;   // position of the new token; context = d_len + 1
-    int H, Hkv, max_ctx, cs, rows;
+    const float* q;  // [nb][H*dh] post-RoPE queries, fp32
+    const bf16* kc[kMaxDecodeBatch];  // layer bases [Hkv][max_ctx][dh] (the new rows are read directly)
+    const bf16* vc[kMaxDecodeBatch];
+    const int* d_len[kMaxDecodeBatch];  // positions of the new tokens; context = d_len + 1
+    int nb, H, Hkv, max_ctx, cs, rows;
     float scale_log2;
-    bf16* out;          // [H*dh]
+    bf16* out;  // [nb][H*dh]
     unsigned* status;
 };
 bool plan_decode_attention_tc(int dh, int group, int Hkv, int max_ctx, int* cs, int* rows);
-cudaError_t launch_attn_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, int group, const AttnDecTcParams& p,
-                                  cudaStream_t s, bool pdl);
+cudaError_t launch_attn_decode_tc(const DecKVMaps& maps, int group, const AttnDecTcParams& p, cudaStream_t s,
+                                  bool pdl);
 
 // Decode-attention launch plan for contexts up to max_ctx: cluster size (CTAs per KV head),
 // keys per shared-memory stage and stage count.
@@ -172,7 +181,8 @@ enum : int { kStageDecQKV = 7, kStageDecAttn = 8, kStageDecO = 9, kStageDecGateU
 cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const DecodeWork& w, const bf16* x_in,
                                 bf16* x_out, int num_sms, cudaStream_t stream, const StageHook& hook, bool pdl_first);
 
-// d_len[i] += 1 for i < count (after all layers of a decode step have read their position)
-cudaError_t launch_advance_lengths(int* d_len, int count, cudaStream_t stream);
+// d_len[b][i] += 1 for i < count, b < nb (after all layers of a decode step have read their
+// positions)
+cudaError_t launch_advance_lengths(int* const* d_len, int nb, int count, cudaStream_t stream);
 
 }  // namespace vla

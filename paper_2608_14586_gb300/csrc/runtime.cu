@@ -148,12 +148,17 @@ struct vla_prefix {
     cudaStream_t cur_stream = nullptr;
     cudaEvent_t pending = nullptr;
     // decode graphs
-    bf16 *d_xin = nullptr, *d_xout = nullptr;  // [D] staging vectors of a decode step
+    bf16 *d_xin = nullptr, *d_xout = nullptr;  // [kMaxDecodeBatch][D] staging vectors of a decode step
     cudaStream_t cap_stream = nullptr;
     struct DecodeGraph {
-        const vla_kv* kv;
-        int lb, le;
+        const vla_kv* kv[vla::kMaxDecodeBatch];  // the step's caches, one per sequence
+        int nb, lb, le;
         cudaGraphExec_t exec;
+        bool uses(const vla_kv* k) const {
+            for (int b = 0; b < nb; ++b)
+                if (kv[b] == k) return true;
+            return false;
+        }
     };
     std::vector<DecodeGraph> graphs;
 };
@@ -315,10 +320,12 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
               dmalloc(&p->ws_q, (size_t)T * p->qc) && dmalloc(&p->ws_attn, (size_t)T * p->qc) &&
               dmalloc(&p->ws_xmid, (size_t)T * D) && dmalloc(&p->ws_m, (size_t)T * p->F_pad) &&
               dmalloc(&p->ws_ss_x, (size_t)T * (D / 256)) &&
-              dmalloc(&p->ws_ss_mid, (size_t)T * (D / 256)) && dmalloc(&p->dq, (size_t)p->qc) &&
-              dmalloc(&p->d_attn, (size_t)p->qc) && dmalloc(&p->d_xmid, (size_t)D) &&
-              dmalloc(&p->d_m, (size_t)p->F_pad) && dmalloc(&p->d_status, 1) &&
-              dmalloc(&p->d_xin, (size_t)D) && dmalloc(&p->d_xout, (size_t)D);
+              dmalloc(&p->ws_ss_mid, (size_t)T * (D / 256)) && dmalloc(&p->dq, (size_t)vla::kMaxDecodeBatch * p->qc) &&
+              dmalloc(&p->d_attn, (size_t)vla::kMaxDecodeBatch * p->qc) &&
+              dmalloc(&p->d_xmid, (size_t)vla::kMaxDecodeBatch * D) &&
+              dmalloc(&p->d_m, (size_t)vla::kMaxDecodeBatch * p->F_pad) && dmalloc(&p->d_status, 1) &&
+              dmalloc(&p->d_xin, (size_t)vla::kMaxDecodeBatch * D) &&
+              dmalloc(&p->d_xout, (size_t)vla::kMaxDecodeBatch * D);
     if (!ok) {
         cudaGetLastError();
         free_prefix(p);
@@ -412,7 +419,7 @@ vla_status vla_kv_destroy(vla_kv* kv) {
     cudaDeviceSynchronize();
     auto& gs = kv->p->graphs;
     for (size_t i = 0; i < gs.size();) {
-        if (gs[i].kv == kv) {
+        if (gs[i].uses(kv)) {
             cudaGraphExecDestroy(gs[i].exec);
             gs.erase(gs.begin() + i);
         } else {
@@ -639,36 +646,59 @@ vla_status vla_prefix_prefill_to_host(vla_prefix* p, const void* hidden_in, int 
                         static_cast<bf16*>(attr.devicePointer), pinned_dst);
 }
 
-vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_begin, int layer_end, vla_kv* kv,
-                             void* hidden_out, vla_stream stream_) {
-    if (!p || !hidden_in || !hidden_out) return VLA_ERR_INVALID_ARG;
+// One decode step of blocks [layer_begin, layer_end) for nb sequences (hidden_in/out [nb][D],
+// one token each, sequence b in cache kvs[b] at that cache's common length).
+static vla_status decode_impl(vla_prefix* p, const void* hidden_in, int nb, int layer_begin, int layer_end,
+                              vla_kv* const* kvs, void* hidden_out, vla_stream stream_) {
+    if (!p || !hidden_in || !hidden_out || !kvs) return VLA_ERR_INVALID_ARG;
+    if (nb < 1 || nb > vla::kMaxDecodeBatch) return VLA_ERR_SHAPE;
     if (!aligned16(hidden_in) || !aligned16(hidden_out)) return VLA_ERR_INVALID_ARG;
-    int p0 = 0;
-    vla_status st = check_range(p, kv, layer_begin, layer_end, 1, &p0);
-    if (st != VLA_OK) return st;
+    int p0[vla::kMaxDecodeBatch];
+    for (int b = 0; b < nb; ++b) {
+        vla_status st = check_range(p, kvs[b], layer_begin, layer_end, 1, &p0[b]);
+        if (st != VLA_OK) return st;
+        for (int c = 0; c < b; ++c)
+            if (layer_begin < layer_end && kvs[c] == kvs[b]) return VLA_ERR_INVALID_ARG;  // one token per cache
+        if (layer_begin < layer_end &&
+            (kvs[b]->max_ctx != kvs[0]->max_ctx || kvs[b]->lb != kvs[0]->lb))  // one plane stride and plan
+            return VLA_ERR_SHAPE;
+    }
     p->last_launches = 0;
     cudaStream_t stream = (cudaStream_t)stream_;
     const int D = p->cfg.hidden;
+    const size_t vec_bytes = (size_t)nb * D * 2;
     if (layer_begin == layer_end) {
         if (hidden_in == hidden_out) return VLA_OK;
-        return cuda_status(cudaMemcpyAsync(hidden_out, hidden_in, (size_t)D * 2, cudaMemcpyDeviceToDevice, stream));
+        return cuda_status(cudaMemcpyAsync(hidden_out, hidden_in, vec_bytes, cudaMemcpyDeviceToDevice, stream));
     }
-    vla::DecodeDims dims = {D, p->cfg.n_heads, p->cfg.n_kv_heads, p->cfg.head_dim, p->F_pad, kv->max_ctx,
+    const vla_kv* kv0 = kvs[0];
+    vla::DecodeDims dims = {D, p->cfg.n_heads, p->cfg.n_kv_heads, p->cfg.head_dim, p->F_pad, kv0->max_ctx,
                             p->cfg.rms_eps};
-    vla::DecodeWork w = {p->dq,      p->d_attn,  p->d_xmid,  p->d_m,      p->rope,
-                         p->d_status, kv->attn_tc, kv->attn_cs, kv->attn_cap, kv->attn_stages};
+    vla::DecodeWork w = {p->dq,       p->d_attn,   p->d_xmid,    p->d_m,        p->rope,
+                         p->d_status, kv0->attn_tc, kv0->attn_cs, kv0->attn_cap, kv0->attn_stages};
     const int nl = layer_end - layer_begin;
     // enqueue the whole step on stream s, reading x_in and chaining through x_out
     auto enqueue = [&](const bf16* x_in, bf16* x_out, cudaStream_t s, const vla::StageHook& hook) {
         cudaError_t e = cudaSuccess;
         for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
             const LayerDev& ld = p->layers[l];
-            vla::DecodeLayer L = {ld.w_qkv, ld.w_o, ld.w_gu, ld.w_d, kv->k_plane(l), kv->v_plane(l),
-                                  kv->d_len + (l - kv->lb)};
+            vla::DecodeLayer L = {};
+            L.w_qkv = ld.w_qkv;
+            L.w_o = ld.w_o;
+            L.w_gu = ld.w_gu;
+            L.w_d = ld.w_d;
+            L.nb = nb;
+            for (int b = 0; b < nb; ++b) {
+                L.kcache[b] = kvs[b]->k_plane(l);
+                L.vcache[b] = kvs[b]->v_plane(l);
+                L.d_len[b] = kvs[b]->d_len + (l - kvs[b]->lb);
+            }
             e = vla::launch_decode_layer(L, dims, w, l == layer_begin ? x_in : x_out, x_out, p->num_sms, s, hook,
                                          l > layer_begin);
         }
-        if (e == cudaSuccess) e = vla::launch_advance_lengths(kv->d_len + (layer_begin - kv->lb), nl, s);
+        int* lens[vla::kMaxDecodeBatch];
+        for (int b = 0; b < nb; ++b) lens[b] = kvs[b]->d_len + (layer_begin - kvs[b]->lb);
+        if (e == cudaSuccess) e = vla::launch_advance_lengths(lens, nb, nl, s);
         return e;
     };
     cudaError_t e = cudaSuccess;
@@ -679,8 +709,12 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
         e = enqueue((const bf16*)hidden_in, (bf16*)hidden_out, stream, hook);
     } else {
         cudaGraphExec_t exec = nullptr;
-        for (const auto& g : p->graphs)
-            if (g.kv == kv && g.lb == layer_begin && g.le == layer_end) exec = g.exec;
+        for (const auto& g : p->graphs) {
+            if (g.nb != nb || g.lb != layer_begin || g.le != layer_end) continue;
+            bool same = true;
+            for (int b = 0; b < nb; ++b) same = same && g.kv[b] == kvs[b];
+            if (same) exec = g.exec;
+        }
         if (!exec) {
             if (!p->cap_stream && cudaStreamCreateWithFlags(&p->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
                 return VLA_ERR_CUDA;
@@ -701,17 +735,38 @@ vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_beg
                 cudaGraphExecDestroy(p->graphs.front().exec);
                 p->graphs.erase(p->graphs.begin());
             }
-            p->graphs.push_back({kv, layer_begin, layer_end, exec});
+            vla_prefix::DecodeGraph g = {};
+            for (int b = 0; b < nb; ++b) g.kv[b] = kvs[b];
+            g.nb = nb;
+            g.lb = layer_begin;
+            g.le = layer_end;
+            g.exec = exec;
+            p->graphs.push_back(g);
         }
-        e = cudaMemcpyAsync(p->d_xin, hidden_in, (size_t)D * 2, cudaMemcpyDeviceToDevice, stream);
+        e = cudaMemcpyAsync(p->d_xin, hidden_in, vec_bytes, cudaMemcpyDeviceToDevice, stream);
         if (e == cudaSuccess) e = cudaGraphLaunch(exec, stream);
-        if (e == cudaSuccess)
-            e = cudaMemcpyAsync(hidden_out, p->d_xout, (size_t)D * 2, cudaMemcpyDeviceToDevice, stream);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(hidden_out, p->d_xout, vec_bytes, cudaMemcpyDeviceToDevice, stream);
     }
     if (e != cudaSuccess) return VLA_ERR_CUDA;
-    for (int l = layer_begin; l < layer_end; ++l) kv->len[l - kv->lb] = p0 + 1;
+    for (int b = 0; b < nb; ++b)
+        for (int l = layer_begin; l < layer_end; ++l) kvs[b]->len[l - kvs[b]->lb] = p0[b] + 1;
     p->last_launches = 5 * nl + 1;
     return VLA_OK;
+}
+
+vla_status vla_prefix_decode(vla_prefix* p, const void* hidden_in, int layer_begin, int layer_end, vla_kv* kv,
+                             void* hidden_out, vla_stream stream) {
+    if (layer_begin == layer_end) {  // a copy: no cache needed
+        if (!p || !hidden_in || !hidden_out) return VLA_ERR_INVALID_ARG;
+        vla_kv* none = nullptr;
+        return decode_impl(p, hidden_in, 1, layer_begin, layer_end, &none, hidden_out, stream);
+    }
+    return decode_impl(p, hidden_in, 1, layer_begin, layer_end, &kv, hidden_out, stream);
+}
+
+vla_status vla_prefix_decode_batch(vla_prefix* p, const void* hidden_in, int batch, int layer_begin, int layer_end,
+                                   vla_kv* const* kvs, void* hidden_out, vla_stream stream) {
+    return decode_impl(p, hidden_in, batch, layer_begin, layer_end, kvs, hidden_out, stream);
 }
 
 vla_status vla_boundary_to_host(const void* hidden_out, int n_tokens, int hidden, void* pinned_dst,

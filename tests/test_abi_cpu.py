@@ -60,6 +60,7 @@ def test_host_side_argument_errors(lib):
     assert lib.vla_prefix_prefill(None, None, 1, 0, 1, None, None, None) == 1
     assert lib.vla_prefix_decode(None, None, 0, 1, None, None, None) == 1
     assert lib.vla_prefix_prefill_to_host(None, None, 1, 0, 1, None, None, None, None) == 1
+    assert lib.vla_prefix_decode_batch(None, None, 2, 0, 1, None, None, None) == 1
     assert lib.vla_boundary_to_host(None, 1, 1, None, None, None, None) == 1
     assert lib.vla_op_gemm_bf16(None, None, 1, 1, 1, None, None) == 1
     assert lib.vla_last_async_error(None) == 1
