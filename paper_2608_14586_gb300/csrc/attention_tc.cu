@@ -37,10 +37,14 @@ struct AttnCfg {
     static constexpr uint32_t Q_BYTES = KCH * CHUNK;
     static constexpr uint32_t KV_BYTES = KCH * CHUNK;
     static constexpr uint32_t P_BYTES = 2 * CHUNK;       // 128 keys = 2 chunks of 64
+    // K is needed one block before V (S = QK^T precedes PV), so K gets the deeper ring; one P
+    // tile suffices because PV(j) is issued as soon as P(j) is written
+    static constexpr int K_STAGES = 3;
+    static constexpr int V_STAGES = 2;
     static constexpr uint32_t OFF_K = Q_BYTES;
-    static constexpr uint32_t OFF_V = OFF_K + 2 * KV_BYTES;
-    static constexpr uint32_t OFF_P = OFF_V + 2 * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_P + 2 * P_BYTES;
+    static constexpr uint32_t OFF_V = OFF_K + K_STAGES * KV_BYTES;
+    static constexpr uint32_t OFF_P = OFF_V + V_STAGES * KV_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
     static constexpr uint32_t SMEM = OFF_BAR + 256 + 1024;
     static constexpr uint32_t TMEM_COLS = 512;           // S0 [0,128) S1 [128,256) O [256, 256+DH)
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(kBM, kBN);
@@ -48,8 +52,8 @@ struct AttnCfg {
 };
 
 struct Bars {
-    uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2], p_full[2], p_free[2],
-        o_final, mma_done;
+    uint64_t q_full, k_full[3], k_empty[3], v_full[2], v_empty[2], s_full[2], s_free[2], p_full, p_free, o_final,
+        mma_done;
     uint32_t tmem_slot;
 };
 
@@ -83,8 +87,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int num_m = (a.M + kBM - 1) / kBM;
-    const int mt = num_m - 1 - (int)blockIdx.x;  // heavy (late) query tiles first
-    const int h = blockIdx.y;
+    // CTAs launch x-fastest: every head of the heaviest (latest) query tile first, then the
+    // next, so the long causal tiles start early and the short ones fill in (longest first)
+    const int mt = num_m - 1 - (int)blockIdx.y;
+    const int h = blockIdx.x;
     const int g = h / (a.H / a.Hkv);
     const int m0 = mt * kBM;
     const int key_end = a.pos0 + min(m0 + kBM, a.M);
@@ -92,16 +98,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (threadIdx.x == 0) {
         mbar_init(&bars->q_full, 1);
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::K_STAGES; ++b) {
             mbar_init(&bars->k_full[b], 1);
             mbar_init(&bars->k_empty[b], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->v_full[b], 1);
             mbar_init(&bars->v_empty[b], 1);
             mbar_init(&bars->s_full[b], 1);
             mbar_init(&bars->s_free[b], 128);
-            mbar_init(&bars->p_full[b], 128);
-            mbar_init(&bars->p_free[b], 1);
         }
+        mbar_init(&bars->p_full, 128);
+        mbar_init(&bars->p_free, 1);
         mbar_init(&bars->o_final, 1);
         mbar_init(&bars->mma_done, 1);
         s_abort = 0;
@@ -136,8 +144,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             while (jk < nblk || jv < nblk) {
                 bool progressed = false;
                 if (jk < nblk) {
-                    const int b = jk & 1;
-                    const uint32_t n = (uint32_t)(jk >> 1);
+                    const int b = jk % C::K_STAGES;
+                    const uint32_t n = (uint32_t)(jk / C::K_STAGES);
                     if (mbar_try_wait(&bars->k_empty[b], (n & 1u) ^ 1u)) {
                         mbar_arrive_expect_tx(&bars->k_full[b], C::KV_BYTES);
                         for (int c = 0; c < C::KCH; ++c)
@@ -174,10 +182,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) {
                 s_abort = 1;
                 set_status(a.status, kDevTimeout);
-                for (int b = 0; b < 2; ++b) {
+                for (int b = 0; b < C::K_STAGES; ++b)
                     if (issued_k & (1u << b)) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
+                for (int b = 0; b < 2; ++b)
                     if (issued_v & (1u << b)) mbar_wait(&bars->v_full[b], (ph_v >> b) & 1u);
-                }
             }
         }
     } else if (warp == 1) {
@@ -188,10 +196,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             auto issue_pv = [&](int i) -> bool {
                 const int bi = i & 1;
                 const uint32_t ni = (uint32_t)(i >> 1);
-                if (!wait_ab(&bars->p_full[bi], ni & 1u, &s_abort)) return false;
+                if (!wait_ab(&bars->p_full, (uint32_t)i & 1u, &s_abort)) return false;
                 if (!wait_ab(&bars->v_full[bi], ni & 1u, &s_abort)) return false;
                 tc_fence_after();
-                const uint32_t sP = smem_u32(smem + C::OFF_P + bi * C::P_BYTES);
+                const uint32_t sP = smem_u32(smem + C::OFF_P);
                 const uint32_t sV = smem_u32(smem + C::OFF_V + bi * C::KV_BYTES);
 #pragma unroll
                 for (int kk = 0; kk < kBN / 16; ++kk) {
@@ -199,20 +207,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
                     umma_bf16_ss(tmem + 256, ad, bd, C::IDESC_O, (i > 0 || kk > 0) ? 1u : 0u);
                 }
-                umma_commit(&bars->p_free[bi]);
+                umma_commit(&bars->p_free);
                 umma_commit(&bars->v_empty[bi]);
                 return true;
             };
             for (int j = 0; j < nblk && ok; ++j) {
                 const int b = j & 1;
                 const uint32_t n = (uint32_t)(j >> 1);
-                if (!wait_ab(&bars->k_full[b], n & 1u, &s_abort) ||
+                const int kb = j % C::K_STAGES;
+                if (!wait_ab(&bars->k_full[kb], (uint32_t)(j / C::K_STAGES) & 1u, &s_abort) ||
                     !wait_ab(&bars->s_free[b], (n & 1u) ^ 1u, &s_abort)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sK = smem_u32(smem + C::OFF_K + b * C::KV_BYTES);
+                const uint32_t sK = smem_u32(smem + C::OFF_K + kb * C::KV_BYTES);
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk) {
                     const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
@@ -220,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     umma_bf16_ss(tmem + b * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
                 }
                 umma_commit(&bars->s_full[b]);
-                umma_commit(&bars->k_empty[b]);
+                umma_commit(&bars->k_empty[kb]);
                 if (j >= 1 && !issue_pv(j - 1)) ok = false;
             }
             if (ok && !issue_pv(nblk - 1)) ok = false;
@@ -260,9 +269,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (key > qpos || key >= a.ctx) sr[i] = 0xFF800000u;  // -inf
                 }
             }
-            float mraw = __uint_as_float(sr[0]);
+            // row max in 8 independent chains (the single softmax warp of each sub-partition has
+            // nothing else to issue meanwhile), then combined
+            float mc[8];
 #pragma unroll
-            for (int i = 1; i < kBN; ++i) mraw = fmaxf(mraw, __uint_as_float(sr[i]));
+            for (int j = 0; j < 8; ++j) mc[j] = __uint_as_float(sr[j]);
+#pragma unroll
+            for (int i = 8; i < kBN; ++i) mc[i & 7] = fmaxf(mc[i & 7], __uint_as_float(sr[i]));
+            const float mraw = fmaxf(fmaxf(fmaxf(mc[0], mc[1]), fmaxf(mc[2], mc[3])),
+                                     fmaxf(fmaxf(mc[4], mc[5]), fmaxf(mc[6], mc[7])));
             const float mx = mraw * a.scale_log2;  // scale > 0
             float m_new = m_run;
             bool need = false;
@@ -276,12 +291,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             l_run *= corr;
             const bool warp_need = __any_sync(0xFFFFFFFFu, need);
             // the P buffer of block j was last read by PV(j-2)
-            if (j >= 2) ok = wait_ab(&bars->p_free[b], (n - 1) & 1u, &s_abort);
+            // the P tile was last read by PV(j-1)
+            if (j >= 1) ok = wait_ab(&bars->p_free, (uint32_t)(j - 1) & 1u, &s_abort);
             if (!__all_sync(0xFFFFFFFFu, ok)) break;
             // P = exp2(s * scale - m) -> bf16 in the 128-byte-swizzled K-major tile
-            uint8_t* prow = smem + C::OFF_P + b * C::P_BYTES + row * 128;
+            uint8_t* prow = smem + C::OFF_P + row * 128;
             const float neg_m = -m_new;
-            float lsum = 0.f;
+            float ls[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums of the row
 #pragma unroll
             for (int c = 0; c < kBN / 8; ++c) {  // 16-byte chunks of 8 keys
                 uint32_t pk[4];
@@ -289,19 +305,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int t = 0; t < 4; ++t) {
                     const float p0 = ex2_approx(fmaf(__uint_as_float(sr[8 * c + 2 * t]), a.scale_log2, neg_m));
                     const float p1 = ex2_approx(fmaf(__uint_as_float(sr[8 * c + 2 * t + 1]), a.scale_log2, neg_m));
-                    lsum += p0 + p1;
+                    ls[t] += p0 + p1;
                     pk[t] = pack_bf16x2(p0, p1);
                 }
                 // keys [8c, 8c+8): 64-key half c/8, 16-byte chunk c%8, swizzled by the row
                 uint8_t* half = prow + (c >> 3) * C::CHUNK;
                 *reinterpret_cast<uint4*>(half + (((c & 7) ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
             }
-            l_run += lsum;
+            l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
             tc_fence_before();
             mbar_arrive(&bars->s_free[b]);
             if (warp_need) {
                 // O must hold PV(j-1) before it is rescaled
-                ok = wait_ab(&bars->p_free[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, &s_abort);
+                ok = wait_ab(&bars->p_free, (uint32_t)(j - 1) & 1u, &s_abort);
                 if (!__all_sync(0xFFFFFFFFu, ok)) break;
                 tc_fence_after();
 #pragma unroll 1
@@ -315,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            mbar_arrive(&bars->p_full[b]);
+            mbar_arrive(&bars->p_full);
             m_run = m_new;
         }
         if (ok) ok = wait_ab(&bars->o_final, 0, &s_abort);
@@ -379,7 +395,7 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
     a.scale_log2 = p.scale_log2;
     a.out = p.out;
     a.status = status;
-    dim3 grid((p.M + kBM - 1) / kBM, p.H);
+    dim3 grid(p.H, (p.M + kBM - 1) / kBM);
     return launch_ex(attn_prefill_tc_kernel<DH>, grid, dim3(kThreads), C::SMEM, stream, pdl, tq, tk, tv, a);
 }
 
