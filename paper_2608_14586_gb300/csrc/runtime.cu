@@ -94,16 +94,8 @@ static int device_sm_count() {
 
 namespace {
 
-constexpr int kBN = 256;  // N tile of the prefill GEMMs (the QKV GEMM may use 128, below)
+constexpr int kBN = 256;  // N tile of every prefill GEMM
 
-// 256 or 128: the N tile that finishes a GEMM of M x N output in fewer SM waves, counting a
-// 128-wide tile as 0.55 of a 256-wide one (half the MMAs plus fixed per-tile cost).
-int gemm_tile_width(int M, int N, int sms) {
-    const int m_tiles = (M + 127) / 128;
-    const int w256 = (m_tiles * ((N + 255) / 256) + sms - 1) / sms;
-    const int w128 = (m_tiles * ((N + 127) / 128) + sms - 1) / sms;
-    return (0.55 * w128 < 1.0 * w256) ? 128 : 256;
-}
 
 // A decode step is ~6 kernels per block (~97 for 16 blocks), each only a few to a few tens
 // of microseconds long, so host launch cost would dominate. The step is captured once per
@@ -115,7 +107,6 @@ constexpr int kMaxDecodeGraphs = 8;
 struct LayerDev {
     bf16 *w_qkv, *w_o, *w_gu, *w_d;
     CUtensorMap tm_qkv, tm_o, tm_gu, tm_d;
-    CUtensorMap tm_qkv128;  // W_qkv with 128-row boxes (QKV GEMM with 128-column tiles)
 };
 
 }  // namespace
@@ -349,7 +340,6 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         e = vla::launch_repack(s, d, D, H, Hkv, dh, cfg->ffn, p->F_pad, 0);
         if (e != cudaSuccess) break;
         if (!vla::make_tmap_bf16(&ld.tm_qkv, ld.w_qkv, p->qkv_n, D, D, kBN) ||
-            !vla::make_tmap_bf16(&ld.tm_qkv128, ld.w_qkv, p->qkv_n, D, D, 128) ||
             !vla::make_tmap_bf16(&ld.tm_o, ld.w_o, D, p->qc, p->qc, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_gu, ld.w_gu, 2 * p->F_pad, D, D, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_d, ld.w_d, D, p->F_pad, p->F_pad, kBN)) {
@@ -509,9 +499,6 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         first_launch = false;
         return r;
     };
-    // QKV tile width: 128 columns when that needs fewer 256-column-equivalent waves (short
-    // frames: at M = 1024 the 256-wide grid is 1.26 waves of 152 SMs, the 128-wide one 2.5)
-    const int qkv_bn = gemm_tile_width(M, p->qkv_n, p->num_sms);
     for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
         const LayerDev& ld = p->layers[l];
         const bf16* x = (l == layer_begin) ? (const bf16*)hidden_in : (const bf16*)hidden_out;
@@ -546,8 +533,8 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ep.len_value = p0 + M;
         ep.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_QKV, true);
-        e = vla::launch_gemm(vla::kEpiQKV, qkv_bn, tm_x, qkv_bn == 128 ? ld.tm_qkv128 : ld.tm_qkv, M, p->qkv_n, D, ep,
-                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_QKV));
+        e = vla::launch_gemm(vla::kEpiQKV, kBN, tm_x, ld.tm_qkv, M, p->qkv_n, D, ep, p->num_sms, stream,
+                             pdl(VLA_STAGE_GEMM_QKV));
         stage_mark(p, VLA_STAGE_GEMM_QKV, false);
         if (e != cudaSuccess) break;
         // causal GQA attention over the cache
