@@ -38,6 +38,7 @@ DECODE_WORKLOAD = "7b_decode16_ctx2304"
 PIPELINE_WORKLOAD = "7b_pipeline32_3072tok"
 BLOCK_WORKLOAD = "7b_block_1024tok"
 PIPELINE_SPLITS = (8, 16, 24)
+HYBRID_SPLIT = 31  # GPU blocks [0, 31), the last block on the host cores
 
 
 def _peaks():
@@ -179,6 +180,8 @@ def cpu_threads() -> int:
     for v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
         if os.environ.get(v, "").isdigit():
             return int(os.environ[v])
+    if hasattr(os, "sched_getaffinity"):
+        return len(os.sched_getaffinity(0))
     return os.cpu_count() or 1
 
 
@@ -243,6 +246,54 @@ def _dec_gateup(dstages: dict, s, D: int) -> dict | None:
     return {"kernel": "gemv_kernel<kGemvSwiGLU> (gate/up + SwiGLU)", "bytes_per_launch": nbytes,
             "avg_launch_us": us, "achieved_gbs": nbytes / (us * 1e-6) / 1e9, "traffic": _traffic("dec_gateup"),
             "timing": "stage-timed pass: plain launches, without the graph's programmatic overlap"}
+
+
+def hybrid_pipeline(vla, p, s, pwl, xs, stream, seed: int, k: int, torch) -> dict:
+    """Frames of the pipeline workload through vla_pipeline (GPU blocks [0, k), CPU blocks
+    [k, N)); per-frame T_G, T_X, T_C (Eq. 12-14) and the steady interval between frames."""
+    D, N, Mp = s.hidden, pwl.n_layers, pwl.n_tokens
+    threads = cpu_threads()
+    t0 = time.perf_counter()
+    cfg = vla.VlaConfig(hidden=D, n_heads=s.n_heads, n_kv_heads=s.n_kv_heads, head_dim=s.head_dim, ffn=s.ffn,
+                        rms_eps=s.rms_eps, rope_base=s.rope_base, max_ctx=Mp)
+    cpu = vla.vla_cpu_model_create(cfg, [synth.layer_weights(s, seed, l) for l in range(k, N)], k, threads)
+    t_create = time.perf_counter() - t0
+    pl = vla.vla_pipeline_create(p, cpu, Mp, 2)
+    res = []
+    try:
+        f = 0
+        while len(res) < len(xs):
+            while f < len(xs):
+                try:
+                    vla.vla_pipeline_submit(pl, f, xs[f], Mp, k, stream)
+                except vla.VlaError as e:
+                    if e.name != "VLA_ERR_BUSY":
+                        raise
+                    break
+                f += 1
+            out = np.empty((Mp, D), dtype=np.uint16)
+            fid, t = vla.vla_pipeline_collect(pl, out, 600000)
+            assert fid == len(res)
+            res.append(t.as_dict())
+    finally:
+        vla.vla_pipeline_destroy(pl)
+        vla.vla_cpu_model_destroy(cpu)
+    tg = statistics.median(r["t_gpu_ms"] for r in res)
+    tx = statistics.median(r["t_xfer_ms"] for r in res)
+    tc = statistics.median(r["t_cpu_ms"] for r in res)
+    done = [r["t_done_s"] for r in res]
+    interval = statistics.median(b - a for a, b in zip(done[1:-1], done[2:])) * 1e3 if len(done) > 2 else None
+    waits = [(r["t_ready_s"] - r["t_start_s"]) * 1e3 for r in res[1:]]
+    block_flops = 2.0 * Mp * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
+                              D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * Mp * Mp * s.head_dim * s.n_heads
+    return {"split": k, "gpu_blocks": k, "cpu_blocks": N - k, "frames": len(res), "tokens": Mp,
+            "t_gpu_ms": tg, "t_xfer_ms": tx, "t_cpu_ms": tc,
+            "steady_interval_ms": interval, "eq14_max_ms": max(tg, tx + tc), "eq12_serial_ms": tg + tx + tc,
+            "cpu_wait_for_gpu_ms": waits,
+            "cpu_suffix_gflops": block_flops * (N - k) / (tc * 1e-3) / 1e9, "cpu_threads": threads,
+            "cpu_model_create_s": t_create,
+            "note": "depth-2 ring; interval = median gap between consecutive frame completions after the "
+                    "first two; the CPU suffix is the library's C++ block on the host cores"}
 
 
 def run_ours(args, dist: Dist):
@@ -591,6 +642,11 @@ def run_ours(args, dist: Dist):
                     "note": "wall time per frame of the GPU prefix with the boundary copy to pinned host memory "
                             "overlapped on a side stream, vs the prefix alone",
                     "splits": splits}
+
+        # ---- hybrid pipeline (Sec. IV-C, Eq. 12-14): GPU prefix [0, k) of frame t+1 while the
+        # host cores run the suffix [k, 32) of frame t, frames handed over in order
+        if not args.no_hybrid:
+            pipeline["hybrid"] = hybrid_pipeline(vla, p, s, pwl, xs, main, seed, HYBRID_SPLIT, torch)
     clock_info = clocks.stop()
 
     # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame
@@ -661,6 +717,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-pipeline", action="store_true")
     ap.add_argument("--no-block1k", action="store_true")
+    ap.add_argument("--no-hybrid", action="store_true", help="skip the GPU prefix + CPU suffix pipeline")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -48,7 +48,8 @@ typedef enum {
     VLA_ERR_OOM = 6,         /* device or pinned allocation failed                   */
     VLA_ERR_CUDA = 7,        /* a CUDA runtime/driver call failed                    */
     VLA_ERR_TIMEOUT = 8,     /* a device-side bounded wait ran out                   */
-    VLA_ERR_UNSUPPORTED = 9  /* model shape outside the supported set                */
+    VLA_ERR_UNSUPPORTED = 9, /* model shape outside the supported set                */
+    VLA_ERR_BUSY = 10        /* every pipeline slot is in flight (vla_cpu.h)         */
 } vla_status;
 
 /* Model shape. Supported: head_dim in {64, 128}; n_heads % n_kv_heads == 0 with
@@ -96,6 +97,10 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
 
 /* Frees everything the object owns. Synchronises the device first. NULL is a no-op. */
 vla_status vla_prefix_destroy(vla_prefix* p);
+
+/* The shape `p` was created with and its block count. Either output may be NULL.
+ * Errors: INVALID_ARG (p NULL). */
+vla_status vla_prefix_info(const vla_prefix* p, vla_config* cfg, int* layer_count);
 
 /* KV cache for blocks [layer_begin, layer_end) of `p`, up to max_ctx positions per layer
  * (max_ctx <= cfg.max_ctx). Layout per layer: K plane then V plane, each

@@ -1,4 +1,5 @@
-"""GB300 LLM-prefix library: Python binding of the C ABI in ``include/vla_prefix.h``.
+"""GB300 LLM-prefix library: Python binding of the C ABI in ``include/vla_prefix.h``,
+``include/vla_ops.h`` and ``include/vla_cpu.h`` (CPU suffix and cross-frame pipeline).
 
 Argument marshalling only: every stage of the prefix forward runs in the CUDA kernels of
 ``libvla_prefix.so`` (built in-tree from ``csrc/`` by ``build()``). Tensors are passed as
@@ -20,7 +21,11 @@ __all__ = [
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
     "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_prefix_decode_batch", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
-    "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "STATUS", "STAGES",
+    "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "vla_prefix_info", "STATUS", "STAGES",
+    "VlaFrameTimes", "vla_cpu_model_create", "vla_cpu_model_destroy", "vla_cpu_model_threads", "vla_cpu_model_info",
+    "vla_cpu_kv_create", "vla_cpu_kv_destroy", "vla_cpu_kv_reset", "vla_cpu_kv_length", "vla_cpu_kv_data",
+    "vla_cpu_prefill", "vla_pipeline_create", "vla_pipeline_submit", "vla_pipeline_collect",
+    "vla_pipeline_in_flight", "vla_pipeline_destroy",
 ]
 
 # stage ids of vla_prefix_stage_times (VLA_STAGE_* in vla_prefix.h)
@@ -29,7 +34,7 @@ STAGES = ("rowstat", "gemm_qkv", "attn_prefill", "gemm_o", "gemm_gateup", "gemm_
 
 STATUS = {0: "VLA_OK", 1: "VLA_ERR_INVALID_ARG", 2: "VLA_ERR_SHAPE", 3: "VLA_ERR_RANGE", 4: "VLA_ERR_KV_FULL",
           5: "VLA_ERR_NOT_PINNED", 6: "VLA_ERR_OOM", 7: "VLA_ERR_CUDA", 8: "VLA_ERR_TIMEOUT",
-          9: "VLA_ERR_UNSUPPORTED"}
+          9: "VLA_ERR_UNSUPPORTED", 10: "VLA_ERR_BUSY"}
 
 
 class VlaError(RuntimeError):
@@ -50,6 +55,17 @@ _WNAMES = ("w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down", "g_attn", "g_
 
 class VlaLayerWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in _WNAMES]
+
+
+class VlaFrameTimes(ctypes.Structure):
+    """Per-frame stage times of the pipeline (vla_frame_times): T_G, T_X, T_C of Eq. 12-14."""
+    _fields_ = [("t_gpu_ms", ctypes.c_double), ("t_xfer_ms", ctypes.c_double), ("t_cpu_ms", ctypes.c_double),
+                ("t_submit_s", ctypes.c_double), ("t_start_s", ctypes.c_double), ("t_ready_s", ctypes.c_double),
+                ("t_done_s", ctypes.c_double),
+                ("split", ctypes.c_int), ("n_tokens", ctypes.c_int)]
+
+    def as_dict(self) -> dict:
+        return {n: getattr(self, n) for n, _ in self._fields_}
 
 
 _lib = None
@@ -94,6 +110,23 @@ def load():
         "vla_prefix_set_timing": ([P, ctypes.c_uint], I),
         "vla_op_attention_decode_noalloc": ([V, V, V, I, I, I, I, I, V, V], I),
         "vla_prefix_stage_times": ([P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int), I], I),
+        "vla_prefix_info": ([P, ctypes.POINTER(VlaConfig), ctypes.POINTER(I)], I),
+        "vla_cpu_model_create": ([ctypes.POINTER(VlaConfig), ctypes.POINTER(VlaLayerWeights), I, I, I,
+                                  ctypes.POINTER(P)], I),
+        "vla_cpu_model_destroy": ([P], I),
+        "vla_cpu_model_threads": ([P], I),
+        "vla_cpu_model_info": ([P, ctypes.POINTER(VlaConfig), ctypes.POINTER(I), ctypes.POINTER(I)], I),
+        "vla_cpu_kv_create": ([P, I, I, I, ctypes.POINTER(P)], I),
+        "vla_cpu_kv_destroy": ([P], I),
+        "vla_cpu_kv_reset": ([P], I),
+        "vla_cpu_kv_length": ([P], I),
+        "vla_cpu_kv_data": ([P, I, ctypes.POINTER(P), ctypes.POINTER(P)], I),
+        "vla_cpu_prefill": ([P, V, I, I, I, P, V], I),
+        "vla_pipeline_create": ([P, P, I, I, ctypes.POINTER(P)], I),
+        "vla_pipeline_submit": ([P, ctypes.c_int64, V, I, I, V], I),
+        "vla_pipeline_collect": ([P, ctypes.POINTER(ctypes.c_int64), V, I, ctypes.POINTER(VlaFrameTimes)], I),
+        "vla_pipeline_in_flight": ([P], I),
+        "vla_pipeline_destroy": ([P], I),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -110,6 +143,8 @@ def _ptr(x) -> int | None:
         return x
     if hasattr(x, "data_ptr"):
         return x.data_ptr()
+    if hasattr(x, "__array_interface__"):  # numpy array in host memory
+        return x.__array_interface__["data"][0]
     if hasattr(x, "value"):
         return x.value
     raise TypeError(f"cannot take a device pointer of {type(x)}")
@@ -277,3 +312,106 @@ def vla_op_attention_decode_noalloc(q, k_plane, v_plane, ctx: int, n_heads: int,
     _check(load().vla_op_attention_decode_noalloc(_ptr(q), _ptr(k_plane), _ptr(v_plane), ctx, n_heads, n_kv_heads,
                                                   head_dim, max_ctx, _ptr(out), _stream(stream)),
            "vla_op_attention_decode_noalloc")
+
+
+def vla_prefix_info(p) -> tuple:
+    """(VlaConfig, layer_count) of a prefix object."""
+    cfg, n = VlaConfig(), ctypes.c_int()
+    _check(load().vla_prefix_info(p, ctypes.byref(cfg), ctypes.byref(n)), "vla_prefix_info")
+    return cfg, n.value
+
+
+# ---------------------------------------------------------------------------------------
+# CPU suffix and cross-frame pipeline (include/vla_cpu.h)
+# ---------------------------------------------------------------------------------------
+def vla_cpu_model_create(cfg: VlaConfig, layers, layer_begin: int, n_threads: int = 0) -> ctypes.c_void_p:
+    """CPU copy of blocks [layer_begin, layer_begin + len(layers)); ``layers`` holds HOST
+    arrays (numpy uint16 bf16 bit patterns or CPU torch tensors) by weight name."""
+    lib = load()
+    arr = (VlaLayerWeights * len(layers))()
+    keep = []
+    for i, w in enumerate(layers):
+        for n in _WNAMES:
+            a = w[n]
+            if hasattr(a, "__array_interface__") and not a.flags["C_CONTIGUOUS"]:
+                import numpy as np
+                a = np.ascontiguousarray(a)
+            keep.append(a)
+            setattr(arr[i], n, _ptr(a))
+    out = ctypes.c_void_p()
+    _check(lib.vla_cpu_model_create(ctypes.byref(cfg), arr, layer_begin, layer_begin + len(layers), n_threads,
+                                    ctypes.byref(out)), "vla_cpu_model_create")
+    return out
+
+
+def vla_cpu_model_destroy(m):
+    _check(load().vla_cpu_model_destroy(m), "vla_cpu_model_destroy")
+
+
+def vla_cpu_model_threads(m) -> int:
+    return load().vla_cpu_model_threads(m)
+
+
+def vla_cpu_model_info(m) -> tuple:
+    """(VlaConfig, layer_begin, layer_end) of a CPU model."""
+    cfg, a, b = VlaConfig(), ctypes.c_int(), ctypes.c_int()
+    _check(load().vla_cpu_model_info(m, ctypes.byref(cfg), ctypes.byref(a), ctypes.byref(b)), "vla_cpu_model_info")
+    return cfg, a.value, b.value
+
+
+def vla_cpu_kv_create(m, layer_begin: int, layer_end: int, max_ctx: int) -> ctypes.c_void_p:
+    out = ctypes.c_void_p()
+    _check(load().vla_cpu_kv_create(m, layer_begin, layer_end, max_ctx, ctypes.byref(out)), "vla_cpu_kv_create")
+    return out
+
+
+def vla_cpu_kv_destroy(kv):
+    _check(load().vla_cpu_kv_destroy(kv), "vla_cpu_kv_destroy")
+
+
+def vla_cpu_kv_reset(kv):
+    _check(load().vla_cpu_kv_reset(kv), "vla_cpu_kv_reset")
+
+
+def vla_cpu_kv_length(kv) -> int:
+    return load().vla_cpu_kv_length(kv)
+
+
+def vla_cpu_kv_data(kv, layer: int):
+    """Host addresses of a layer's K and V planes [n_kv_heads][max_ctx][head_dim] bf16."""
+    k, v = ctypes.c_void_p(), ctypes.c_void_p()
+    _check(load().vla_cpu_kv_data(kv, layer, ctypes.byref(k), ctypes.byref(v)), "vla_cpu_kv_data")
+    return k.value, v.value
+
+
+def vla_cpu_prefill(m, hidden_in, n_tokens: int, layer_begin: int, layer_end: int, kv, hidden_out):
+    """Blocks [layer_begin, layer_end) on the host; hidden_in / hidden_out are host arrays."""
+    _check(load().vla_cpu_prefill(m, _ptr(hidden_in), n_tokens, layer_begin, layer_end, kv, _ptr(hidden_out)),
+           "vla_cpu_prefill")
+
+
+def vla_pipeline_create(gpu, cpu, max_tokens: int, depth: int = 2) -> ctypes.c_void_p:
+    out = ctypes.c_void_p()
+    _check(load().vla_pipeline_create(gpu, cpu, max_tokens, depth, ctypes.byref(out)), "vla_pipeline_create")
+    return out
+
+
+def vla_pipeline_submit(pl, frame_id: int, hidden_in, n_tokens: int, split: int, stream=None):
+    _check(load().vla_pipeline_submit(pl, frame_id, _ptr(hidden_in), n_tokens, split, _stream(stream)),
+           "vla_pipeline_submit")
+
+
+def vla_pipeline_collect(pl, hidden_out=None, timeout_ms: int = -1) -> tuple:
+    """(frame_id, VlaFrameTimes) of the oldest frame once done; h^(N) copied into hidden_out."""
+    fid, t = ctypes.c_int64(), VlaFrameTimes()
+    _check(load().vla_pipeline_collect(pl, ctypes.byref(fid), _ptr(hidden_out), timeout_ms, ctypes.byref(t)),
+           "vla_pipeline_collect")
+    return fid.value, t
+
+
+def vla_pipeline_in_flight(pl) -> int:
+    return load().vla_pipeline_in_flight(pl)
+
+
+def vla_pipeline_destroy(pl):
+    _check(load().vla_pipeline_destroy(pl), "vla_pipeline_destroy")

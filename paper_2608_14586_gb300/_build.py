@@ -1,8 +1,9 @@
 """Builds ``libvla_prefix.so`` (the C-ABI library) in-tree with nvcc for sm_103a.
 
-Each translation unit under ``csrc/`` compiles in its own nvcc process (in parallel); the
-objects link into one shared library next to this file. Rebuilds only when a source or
-header is newer than the library.
+Each translation unit under ``csrc/`` compiles in its own process (in parallel): the CUDA
+sources with nvcc, the host-only sources (CPU suffix, pipeline runtime) with the host C++
+compiler. The objects link into one shared library next to this file. Rebuilds only when a
+source or header is newer than the library.
 """
 from __future__ import annotations
 
@@ -31,8 +32,24 @@ def nvcc() -> str:
     raise RuntimeError("nvcc not found")
 
 
+# Host code: portable C++ (GCC vector extensions, no ISA-specific flags), the same source on
+# x86-64 and aarch64 hosts.
+CXX_FLAGS = ["-O3", "-std=gnu++17", "-fPIC", "-pthread", "-ffp-contract=fast", "-I", INCLUDE, "-I", CSRC]
+
+
+def cxx() -> str:
+    for cand in (os.environ.get("CXX"), shutil.which("g++"), shutil.which("c++")):
+        if cand and os.path.exists(cand):
+            return cand
+    raise RuntimeError("no host C++ compiler found")
+
+
+def _cuda_include() -> str:
+    return os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(nvcc()))), "include")
+
+
 def _sources():
-    return sorted(glob.glob(os.path.join(CSRC, "*.cu")))
+    return sorted(glob.glob(os.path.join(CSRC, "*.cu"))) + sorted(glob.glob(os.path.join(CSRC, "*.cpp")))
 
 
 def _deps():
@@ -54,12 +71,18 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     cc = nvcc()
     srcs = _sources()
 
+    host_cc = cxx()
+    cuda_inc = _cuda_include()
+
     def compile_one(src):
         obj = os.path.join(OBJDIR, os.path.basename(src) + ".o")
-        cmd = [cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj]
+        if src.endswith(".cpp"):
+            cmd = [host_cc, *CXX_FLAGS, "-I", cuda_inc, "-c", src, "-o", obj]
+        else:
+            cmd = [cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
-            raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+            raise RuntimeError(f"compile failed for {src}:\n{r.stdout}\n{r.stderr}")
         if verbose and (r.stdout or r.stderr):
             print(r.stdout, r.stderr)
         return obj
@@ -67,7 +90,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
     with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, min(len(srcs), os.cpu_count() or 4))) as ex:
         objs = list(ex.map(compile_one, srcs))
     tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart=static"]
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart=static", "-lpthread"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -276,6 +276,7 @@ const char* vla_status_str(vla_status s) {
         case VLA_ERR_CUDA: return "cuda error";
         case VLA_ERR_TIMEOUT: return "device wait timed out";
         case VLA_ERR_UNSUPPORTED: return "unsupported model shape";
+        case VLA_ERR_BUSY: return "all pipeline slots in flight";
     }
     return "unknown status";
 }
@@ -783,6 +784,13 @@ vla_status vla_last_async_error(vla_prefix* p) {
 }
 
 int vla_last_launch_count(const vla_prefix* p) { return p ? p->last_launches : 0; }
+
+vla_status vla_prefix_info(const vla_prefix* p, vla_config* cfg, int* layer_count) {
+    if (!p) return VLA_ERR_INVALID_ARG;
+    if (cfg) *cfg = p->cfg;
+    if (layer_count) *layer_count = p->L;
+    return VLA_OK;
+}
 
 vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask) {
     if (!p) return VLA_ERR_INVALID_ARG;
