@@ -5,17 +5,20 @@
 // projection, QKV + rotary embedding + KV write, causal GQA attention, output projection +
 // residual, RMSNorm, gate/up + SwiGLU, down projection + residual), with bf16 weights and
 // activations, fp32 accumulation and bf16 rounding at the points where the GPU stores bf16:
-//   * projections C = A W^T: W is repacked at create time into panels of 16 output rows,
-//     [panel][k][16] bf16, gains folded in and rounded to bf16 as on the GPU. A 6 x 16
-//     register-blocked fp32 micro-kernel (GCC vector extensions over 128-bit lanes: NEON on
-//     an Arm host, SSE on x86) runs over 256-deep k blocks of a task tile of 48 rows x 128
-//     columns. Every output element's k order is fixed, so results do not depend on how tiles
-//     fall to threads. The epilogues mirror the GPU's: 1/rms scaling, RoPE and the KV write
-//     for QKV; the residual add for O and down; SwiGLU for gate/up, whose rows are grouped as
-//     64 gate rows then the 64 matching up rows so one tile holds both halves of its units;
-//   * attention: one task per (KV head, block of 16 queries), longest first; keys and values
-//     in 64-row blocks converted to fp32, one online softmax in fp32 per query head of the
-//     group; a key block past a query's position is skipped for that query, so each query's
+//   * projections C = A W^T: W is repacked at create time into panels of 8 output rows,
+//     [panel][k][8] bf16, gains folded in and rounded to bf16 as on the GPU. The register
+//     tile is 12 rows x 8 columns: three 4-row vectors of A times each of the 8 weight values
+//     of a k step (24 fp32 vector accumulators; GCC vector extensions over 128-bit lanes: NEON
+//     on an Arm host, SSE on x86). A task tile is 96 rows x 128 columns over 256-deep k
+//     blocks; each k block's weight slice is widened to fp32 once and reused by the tile's
+//     eight 12-row panels. Every output element's k order is fixed, so results do not depend
+//     on how tiles fall to threads. The epilogues mirror the GPU's: 1/rms scaling, RoPE and
+//     the KV write for QKV; the residual add for O and down; SwiGLU for gate/up, whose rows
+//     are grouped as 64 gate rows then the 64 matching up rows so one tile holds both halves;
+//   * attention: one task per (KV head, block of 16 queries), longest first; per 64-key block
+//     the scores and the output update run on the same register tile (S^T = K Q^T, O^T +=
+//     V^T P^T) around an fp32 online softmax; a key past a query's position gets probability
+//     0 and a key block wholly past it leaves that query's state unchanged, so each query's
 //     result does not depend on which other queries share its call (causal invariance);
 //   * a fixed pool of worker threads that draw tasks from an atomic counter; the thread that
 //     makes a compute call works too.
@@ -39,10 +42,10 @@ typedef float v4f __attribute__((vector_size(16)));
 typedef uint16_t v4h __attribute__((vector_size(8)));
 typedef uint32_t v4u __attribute__((vector_size(16)));
 
-constexpr int kMR = 6;    // rows of one micro-tile
-constexpr int kNR = 16;   // columns of one micro-tile = weight rows of one panel
+constexpr int kMR = 12;   // rows of one register tile (three 4-lane vectors)
+constexpr int kNR = 8;    // columns of one register tile = weight rows of one panel
 constexpr int kKC = 256;  // k block
-constexpr int kTM = 48;   // rows of one task tile
+constexpr int kTM = 96;   // rows of one task tile
 constexpr int kTN = 128;  // columns of one task tile
 constexpr int kGU = 64;   // feed-forward units per gate/up tile (64 gate + 64 up columns)
 constexpr int kQB = 16;   // queries per attention task
@@ -150,50 +153,43 @@ struct Packed {
 
 struct Scratch {
     std::vector<float> apack;   // [kTM / kMR][kKC][kMR]
-    std::vector<float> ctile;   // [kTM][kTN]
-    std::vector<float> kf, vf;  // [kKB][dh]
-    std::vector<float> qv, ov;  // [G * kQB][dh]
-    std::vector<float> mx, l;   // [G * kQB]
-    std::vector<float> s;       // [kKB]
+    std::vector<float> bf;      // [kKC][kNR]: one panel's k block widened to fp32
+    std::vector<float> ctile;   // [kTN][kTM], column-major
+    std::vector<float> qpk, kpk, vpk, ppk, st, ot;  // attention operands (see attention())
+    std::vector<float> mx, l;                        // [G * kQB]
 };
 
-// c[MR x 16] (row stride ldc) = (init ? 0 : c) + a-panel x b-panel over kc steps.
-template <int MR>
-inline void micro(const float* a, const uint16_t* b, int kc, float* c, int ldc, bool init) {
-    v4f acc[MR][4];
-    for (int r = 0; r < MR; ++r)
-        for (int i = 0; i < 4; ++i) {
+// c[8 columns][4*MV rows] (column stride ldc) = (init ? 0 : c) + a-panel x b-panel over kc
+// steps; a-panel [k][kMR] fp32 (rows), b-panel [k][kNR] fp32 (columns).
+template <int MV>
+inline void micro(const float* a, const float* b, int kc, float* c, int ldc, bool init) {
+    v4f acc[kNR][MV];
+    for (int j = 0; j < kNR; ++j)
+        for (int i = 0; i < MV; ++i) {
             if (init) {
-                acc[r][i] = v4f{0.f, 0.f, 0.f, 0.f};
+                acc[j][i] = v4f{0.f, 0.f, 0.f, 0.f};
             } else {
-                std::memcpy(&acc[r][i], c + (size_t)r * ldc + 4 * i, sizeof(v4f));
+                std::memcpy(&acc[j][i], c + (size_t)j * ldc + 4 * i, sizeof(v4f));
             }
         }
     for (int k = 0; k < kc; ++k) {
-        const v4f b0 = ld_bf4(b), b1 = ld_bf4(b + 4), b2 = ld_bf4(b + 8), b3 = ld_bf4(b + 12);
-        b += kNR;
-        for (int r = 0; r < MR; ++r) {
-            const float ar = a[r];
-            acc[r][0] += b0 * ar;
-            acc[r][1] += b1 * ar;
-            acc[r][2] += b2 * ar;
-            acc[r][3] += b3 * ar;
-        }
+        v4f av[MV];
+        for (int i = 0; i < MV; ++i) std::memcpy(&av[i], a + 4 * i, sizeof(v4f));
         a += kMR;
+        for (int j = 0; j < kNR; ++j) {
+            const float bj = b[j];
+            for (int i = 0; i < MV; ++i) acc[j][i] += av[i] * bj;
+        }
+        b += kNR;
     }
-    for (int r = 0; r < MR; ++r)
-        for (int i = 0; i < 4; ++i) std::memcpy(c + (size_t)r * ldc + 4 * i, &acc[r][i], sizeof(v4f));
+    for (int j = 0; j < kNR; ++j)
+        for (int i = 0; i < MV; ++i) std::memcpy(c + (size_t)j * ldc + 4 * i, &acc[j][i], sizeof(v4f));
 }
 
-inline void micro_any(int mr, const float* a, const uint16_t* b, int kc, float* c, int ldc, bool init) {
-    switch (mr) {
-        case 6: micro<6>(a, b, kc, c, ldc, init); break;
-        case 5: micro<5>(a, b, kc, c, ldc, init); break;
-        case 4: micro<4>(a, b, kc, c, ldc, init); break;
-        case 3: micro<3>(a, b, kc, c, ldc, init); break;
-        case 2: micro<2>(a, b, kc, c, ldc, init); break;
-        default: micro<1>(a, b, kc, c, ldc, init); break;
-    }
+inline void micro_any(int rows, const float* a, const float* b, int kc, float* c, int ldc, bool init) {
+    if (rows > 8) micro<3>(a, b, kc, c, ldc, init);
+    else if (rows > 4) micro<2>(a, b, kc, c, ldc, init);
+    else micro<1>(a, b, kc, c, ldc, init);
 }
 
 }  // namespace
@@ -213,6 +209,7 @@ struct vla_cpu_model {
     // workspace for cfg.max_ctx tokens
     std::vector<uint16_t> h[2], q, att, xmid, mbuf;
     std::vector<float> rinv;
+    std::vector<float> xrows;  // [4][max K]: the rows of a short (decode) projection in fp32
     ~vla_cpu_model() { delete pool; }
 };
 
@@ -256,10 +253,55 @@ void pack(Pool& pool, Packed& P, int N, int K, RowFn row, const uint16_t* gain) 
     });
 }
 
-// C = A W^T over task tiles; epi(m0, rows, n0, C, ldc) consumes each finished tile.
+// Up to kGemvRows rows (decode): each weight panel streams once, straight from its bf16
+// words, into 2 x R vector accumulators. Every element sees the same sequence of fused
+// multiply-adds as in the tiled path (k ascending from 0), so both give the same bits.
+constexpr int kGemvRows = 4;
+
+template <int R>
+void gemv_panel(const float* x, int K, const uint16_t* bp, float* c, int ldc) {
+    v4f acc[R][2];
+    for (int r = 0; r < R; ++r) acc[r][0] = acc[r][1] = v4f{0.f, 0.f, 0.f, 0.f};
+    for (int k = 0; k < K; ++k) {
+        const v4f w0 = ld_bf4(bp + (size_t)k * kNR), w1 = ld_bf4(bp + (size_t)k * kNR + 4);
+        for (int r = 0; r < R; ++r) {
+            const float xr = x[(size_t)r * K + k];
+            acc[r][0] += w0 * xr;
+            acc[r][1] += w1 * xr;
+        }
+    }
+    for (int r = 0; r < R; ++r)
+        for (int j = 0; j < 4; ++j) {
+            c[(size_t)j * ldc + r] = acc[r][0][j];
+            c[(size_t)(j + 4) * ldc + r] = acc[r][1][j];
+        }
+}
+
+// C = A W^T over task tiles; epi(m0, rows, n0, C, ldc) consumes each finished tile, whose
+// element (row m0 + r, column n0 + n) is C[n * ldc + r].
 template <class Epi>
 void gemm(Model* m, const uint16_t* A, int M, const Packed& B, const Epi& epi) {
     const int K = B.K;
+    if (M <= kGemvRows) {
+        float* x = m->xrows.data();
+        for (size_t i = 0; i < (size_t)M * K; ++i) x[i] = bf2f(A[i]);
+        m->pool->run(B.N / kTN, [&](int t, int tid) {
+            float* C = m->scratch[tid].ctile.data();
+            const int n0 = t * kTN;
+            for (int j = 0; j < kTN / kNR; ++j) {
+                const uint16_t* bp = B.w.data() + (size_t)(n0 / kNR + j) * K * kNR;
+                float* c = C + (size_t)j * kNR * kTM;
+                switch (M) {
+                    case 4: gemv_panel<4>(x, K, bp, c, kTM); break;
+                    case 3: gemv_panel<3>(x, K, bp, c, kTM); break;
+                    case 2: gemv_panel<2>(x, K, bp, c, kTM); break;
+                    default: gemv_panel<1>(x, K, bp, c, kTM); break;
+                }
+            }
+            epi(0, M, n0, C, kTM);
+        });
+        return;
+    }
     const int tm = (M + kTM - 1) / kTM, tn = B.N / kTN;
     m->pool->run(tm * tn, [&](int t, int tid) {
         Scratch& s = m->scratch[tid];
@@ -267,6 +309,7 @@ void gemm(Model* m, const uint16_t* A, int M, const Packed& B, const Epi& epi) {
         const int m0 = im * kTM, rows = std::min(kTM, M - m0), n0 = in * kTN;
         const int np = (rows + kMR - 1) / kMR;
         float* C = s.ctile.data();
+        float* bf = s.bf.data();
         for (int k0 = 0; k0 < K; k0 += kKC) {
             const int kc = std::min(kKC, K - k0);
             for (int p = 0; p < np; ++p) {
@@ -283,14 +326,16 @@ void gemm(Model* m, const uint16_t* A, int M, const Packed& B, const Epi& epi) {
             }
             for (int j = 0; j < kTN / kNR; ++j) {
                 const uint16_t* bp = B.w.data() + ((size_t)(n0 / kNR + j) * K + k0) * kNR;
-                for (int p = 0; p < np; ++p) {
-                    const int mr = std::min(kMR, rows - p * kMR);
-                    micro_any(mr, s.apack.data() + (size_t)p * kKC * kMR, bp, kc, C + (size_t)p * kMR * kTN + j * kNR,
-                              kTN, k0 == 0);
+                for (int e = 0; e < kc * kNR; e += 4) {
+                    const v4f v = ld_bf4(bp + e);
+                    std::memcpy(bf + e, &v, sizeof v);
                 }
+                for (int p = 0; p < np; ++p)
+                    micro_any(rows - p * kMR, s.apack.data() + (size_t)p * kKC * kMR, bf, kc,
+                              C + (size_t)j * kNR * kTM + p * kMR, kTM, k0 == 0);
             }
         }
-        epi(m0, rows, n0, C, kTN);
+        epi(m0, rows, n0, C, kTM);
     });
 }
 
@@ -312,26 +357,36 @@ void row_rinv(Model* m, const uint16_t* x, int M, float* out) {
 }
 
 // Causal GQA attention of M queries at positions p0.. over cache positions [0, p0 + M).
+// Per task (KV head g, block of kQB queries): the G query heads' vectors of the block form
+// nq = G * rows columns. Per 64-key block: S^T = K Q^T and O^T += V^T P^T on the register
+// tile (keys resp. head dims as rows, queries as columns), with the online-softmax update
+// (running max, rescale of the running sum and output) in between. Keys past a query's
+// position get probability 0 and a block wholly past it leaves its state unchanged.
 void attention(Model* m, const uint16_t* q, const uint16_t* kp, const uint16_t* vp, int max_ctx, int p0, int M,
                uint16_t* out) {
     const int H = m->cfg.n_heads, Hkv = m->cfg.n_kv_heads, dh = m->cfg.head_dim, G = H / Hkv;
-    const int nv = dh / 4;
     const float scale = 1.0f / std::sqrt((float)dh);
     const int nqb = (M + kQB - 1) / kQB;
+    const int dpan = (dh + kMR - 1) / kMR;  // head-dim panels of the O tile
     m->pool->run(Hkv * nqb, [&](int t, int tid) {
         Scratch& s = m->scratch[tid];
         const int g = t % Hkv, qb = nqb - 1 - t / Hkv;  // longest query blocks first
         const int r0 = qb * kQB, r1 = std::min(M, r0 + kQB), nr = r1 - r0;
-        const int nq = G * nr;
-        float* qv = s.qv.data();
-        float* ov = s.ov.data();
-        for (int hh = 0; hh < G; ++hh)
-            for (int i = 0; i < nr; ++i) {
-                const uint16_t* src = q + (size_t)(r0 + i) * H * dh + (size_t)(g * G + hh) * dh;
-                float* dst = qv + (size_t)(hh * nr + i) * dh;
-                for (int d = 0; d < dh; ++d) dst[d] = bf2f(src[d]) * scale;
-            }
-        std::fill(ov, ov + (size_t)nq * dh, 0.f);
+        const int nq = G * nr, nqp = (nq + kNR - 1) / kNR;  // query columns, column panels
+        float* qpk = s.qpk.data();  // [nqp][dh][kNR]   queries (scaled), B operand of S
+        float* kpk = s.kpk.data();  // [6][dh][kMR]     keys of the block, A operand of S
+        float* vpk = s.vpk.data();  // [dpan][kKB][kMR] values of the block, A operand of O
+        float* ppk = s.ppk.data();  // [nqp][kKB][kNR]  probabilities, B operand of O
+        float* st = s.st.data();    // [nqp * kNR][kKB] scores, query-major
+        float* ot = s.ot.data();    // [nqp * kNR][dh]  unnormalised outputs, query-major
+        std::fill(qpk, qpk + (size_t)nqp * dh * kNR, 0.f);
+        for (int c = 0; c < nq; ++c) {
+            const int hh = c / nr, i = c % nr;
+            const uint16_t* src = q + (size_t)(r0 + i) * H * dh + (size_t)(g * G + hh) * dh;
+            float* dst = qpk + (size_t)(c / kNR) * dh * kNR + (c % kNR);
+            for (int d = 0; d < dh; ++d) dst[(size_t)d * kNR] = bf2f(src[d]) * scale;
+        }
+        std::fill(ot, ot + (size_t)nqp * kNR * dh, 0.f);
         std::fill(s.mx.begin(), s.mx.begin() + nq, -INFINITY);
         std::fill(s.l.begin(), s.l.begin() + nq, 0.f);
         const int nkeys = p0 + r1;  // keys visible to the block's last query
@@ -339,64 +394,58 @@ void attention(Model* m, const uint16_t* q, const uint16_t* kp, const uint16_t* 
         const uint16_t* vg = vp + (size_t)g * max_ctx * dh;
         for (int kb0 = 0; kb0 < nkeys; kb0 += kKB) {
             const int kn = std::min(kKB, nkeys - kb0);
-            for (int j = 0; j < kn; ++j)
-                for (int d = 0; d < dh; d += 4) {
-                    const v4f a = ld_bf4(kg + (size_t)(kb0 + j) * dh + d), b = ld_bf4(vg + (size_t)(kb0 + j) * dh + d);
-                    std::memcpy(&s.kf[(size_t)j * dh + d], &a, sizeof a);
-                    std::memcpy(&s.vf[(size_t)j * dh + d], &b, sizeof b);
+            const int kpan = (kn + kMR - 1) / kMR;
+            for (int j = 0; j < kpan * kMR; ++j) {
+                float* dst = kpk + (size_t)(j / kMR) * dh * kMR + (j % kMR);
+                if (j < kn) {
+                    const uint16_t* src = kg + (size_t)(kb0 + j) * dh;
+                    for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = bf2f(src[d]);
+                } else {
+                    for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = 0.f;
                 }
-            for (int hh = 0; hh < G; ++hh)
-                for (int i = 0; i < nr; ++i) {
-                    const int qi = hh * nr + i;
-                    const int jn = std::min(kn, p0 + r0 + i - kb0 + 1);  // keys at or before the query
-                    if (jn <= 0) continue;
-                    const float* qq = qv + (size_t)qi * dh;
-                    float smax = -INFINITY;
-                    for (int j = 0; j < jn; ++j) {
-                        const float* kk = s.kf.data() + (size_t)j * dh;
-                        v4f a0 = {0.f, 0.f, 0.f, 0.f}, a1 = a0;
-                        for (int d = 0; d < nv; d += 2) {
-                            v4f x0, x1, y0, y1;
-                            std::memcpy(&x0, qq + 4 * d, 16);
-                            std::memcpy(&x1, qq + 4 * d + 4, 16);
-                            std::memcpy(&y0, kk + 4 * d, 16);
-                            std::memcpy(&y1, kk + 4 * d + 4, 16);
-                            a0 += x0 * y0;
-                            a1 += x1 * y1;
-                        }
-                        const float sc = hsum(a0 + a1);
-                        s.s[j] = sc;
-                        smax = std::max(smax, sc);
-                    }
-                    const float mold = s.mx[qi], mnew = std::max(mold, smax);
-                    const float corr = std::exp(mold - mnew);  // 0 when mold = -inf
-                    float lsum = s.l[qi] * corr;
-                    float* oo = ov + (size_t)qi * dh;
-                    for (int d = 0; d < dh; ++d) oo[d] *= corr;
-                    for (int j = 0; j < jn; ++j) {
-                        const float pj = std::exp(s.s[j] - mnew);
-                        lsum += pj;
-                        const float* vv = s.vf.data() + (size_t)j * dh;
-                        for (int d = 0; d < dh; d += 4) {
-                            v4f o4, v4;
-                            std::memcpy(&o4, oo + d, 16);
-                            std::memcpy(&v4, vv + d, 16);
-                            o4 += v4 * pj;
-                            std::memcpy(oo + d, &o4, 16);
-                        }
-                    }
-                    s.mx[qi] = mnew;
-                    s.l[qi] = lsum;
-                }
-        }
-        for (int hh = 0; hh < G; ++hh)
-            for (int i = 0; i < nr; ++i) {
-                const int qi = hh * nr + i;
-                const float inv = 1.0f / s.l[qi];
-                uint16_t* dst = out + (size_t)(r0 + i) * H * dh + (size_t)(g * G + hh) * dh;
-                const float* oo = ov + (size_t)qi * dh;
-                for (int d = 0; d < dh; ++d) dst[d] = f2bf(oo[d] * inv);
             }
+            for (int j = 0; j < kn; ++j) {
+                const uint16_t* src = vg + (size_t)(kb0 + j) * dh;
+                for (int d = 0; d < dh; ++d) vpk[((size_t)(d / kMR) * kKB + j) * kMR + (d % kMR)] = bf2f(src[d]);
+            }
+            for (int cp = 0; cp < nqp; ++cp)
+                for (int kq = 0; kq < kpan; ++kq)
+                    micro_any(kn - kq * kMR, kpk + (size_t)kq * dh * kMR, qpk + (size_t)cp * dh * kNR, dh,
+                              st + (size_t)cp * kNR * kKB + kq * kMR, kKB, true);
+            std::fill(ppk, ppk + (size_t)nqp * kKB * kNR, 0.f);
+            for (int c = 0; c < nq; ++c) {
+                const int i = c % nr;
+                const int jn = std::min(kn, p0 + r0 + i - kb0 + 1);  // keys at or before the query
+                if (jn <= 0) continue;
+                const float* sc = st + (size_t)c * kKB;
+                float smax = -INFINITY;
+                for (int j = 0; j < jn; ++j) smax = std::max(smax, sc[j]);
+                const float mold = s.mx[c], mnew = std::max(mold, smax);
+                const float corr = std::exp(mold - mnew);  // 0 when mold = -inf
+                float lsum = s.l[c] * corr;
+                float* pc = ppk + (size_t)(c / kNR) * kKB * kNR + (c % kNR);
+                for (int j = 0; j < jn; ++j) {
+                    const float pj = std::exp(sc[j] - mnew);
+                    lsum += pj;
+                    pc[(size_t)j * kNR] = pj;
+                }
+                float* oc = ot + (size_t)c * dh;
+                for (int d = 0; d < dh; ++d) oc[d] *= corr;
+                s.mx[c] = mnew;
+                s.l[c] = lsum;
+            }
+            for (int cp = 0; cp < nqp; ++cp)
+                for (int dp = 0; dp < dpan; ++dp)
+                    micro_any(dh - dp * kMR, vpk + (size_t)dp * kKB * kMR, ppk + (size_t)cp * kKB * kNR, kn,
+                              ot + (size_t)cp * kNR * dh + dp * kMR, dh, false);
+        }
+        for (int c = 0; c < nq; ++c) {
+            const int hh = c / nr, i = c % nr;
+            const float inv = 1.0f / s.l[c];
+            uint16_t* dst = out + (size_t)(r0 + i) * H * dh + (size_t)(g * G + hh) * dh;
+            const float* oc = ot + (size_t)c * dh;
+            for (int d = 0; d < dh; ++d) dst[d] = f2bf(oc[d] * inv);
+        }
     });
 }
 
@@ -424,7 +473,7 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
             for (int r = 0; r < rows; ++r) {
                 const int pos = p0 + m0 + r;
                 const float ri = rinv[m0 + r];
-                const float* cr = C + (size_t)r * ldc + (h0 - n0);
+                const float* cr = C + (size_t)(h0 - n0) * ldc + r;  // column j at cr[j * ldc]
                 uint16_t* dst;
                 if (head < H) dst = q + (size_t)(m0 + r) * qc + (size_t)head * dh;
                 else if (head < H + Hkv) dst = kp + ((size_t)(head - H) * max_ctx + pos) * dh;
@@ -432,12 +481,12 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
                 if (head < H + Hkv) {
                     const float* cs = rope + (size_t)pos * dh;  // (cos, sin) of the pairs j < dh/2
                     for (int j = 0; j < half; ++j) {
-                        const float a = cr[j] * ri, b = cr[j + half] * ri;
+                        const float a = cr[(size_t)j * ldc] * ri, b = cr[(size_t)(j + half) * ldc] * ri;
                         dst[j] = f2bf(a * cs[2 * j] - b * cs[2 * j + 1]);
                         dst[j + half] = f2bf(b * cs[2 * j] + a * cs[2 * j + 1]);
                     }
                 } else {
-                    for (int d = 0; d < dh; ++d) dst[d] = f2bf(cr[d] * ri);
+                    for (int d = 0; d < dh; ++d) dst[d] = f2bf(cr[(size_t)d * ldc] * ri);
                 }
             }
         }
@@ -448,7 +497,7 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
         for (int r = 0; r < rows; ++r) {
             const uint16_t* xr = x + (size_t)(m0 + r) * D + n0;
             uint16_t* dst = xmid + (size_t)(m0 + r) * D + n0;
-            for (int n = 0; n < kTN; ++n) dst[n] = f2bf(bf2f(xr[n]) + C[(size_t)r * ldc + n]);
+            for (int n = 0; n < kTN; ++n) dst[n] = f2bf(bf2f(xr[n]) + C[(size_t)n * ldc + r]);
         }
     });
     // RMSNorm statistics; gate/up + SwiGLU
@@ -459,7 +508,7 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
             const float ri = rinv[m0 + r];
             uint16_t* dst = mb + (size_t)(m0 + r) * F_pad + u0;
             for (int i = 0; i < kGU; ++i) {
-                const float gt = C[(size_t)r * ldc + i] * ri, up = C[(size_t)r * ldc + kGU + i] * ri;
+                const float gt = C[(size_t)i * ldc + r] * ri, up = C[(size_t)(kGU + i) * ldc + r] * ri;
                 dst[i] = f2bf(gt / (1.0f + std::exp(-gt)) * up);
             }
         }
@@ -469,7 +518,7 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
         for (int r = 0; r < rows; ++r) {
             const uint16_t* xr = xmid + (size_t)(m0 + r) * D + n0;
             uint16_t* dst = y + (size_t)(m0 + r) * D + n0;
-            for (int n = 0; n < kTN; ++n) dst[n] = f2bf(bf2f(xr[n]) + C[(size_t)r * ldc + n]);
+            for (int n = 0; n < kTN; ++n) dst[n] = f2bf(bf2f(xr[n]) + C[(size_t)n * ldc + r]);
         }
     });
 }
@@ -523,14 +572,18 @@ vla_status vla_cpu_model_create(const vla_config* cfg, const vla_layer_weights* 
         m->scratch.resize(m->pool->size());
         for (Scratch& s : m->scratch) {
             s.apack.assign((size_t)kTM * kKC, 0.f);
+            s.bf.assign((size_t)kKC * kNR, 0.f);
             s.ctile.assign((size_t)kTM * kTN, 0.f);
-            s.kf.assign((size_t)kKB * dh, 0.f);
-            s.vf.assign((size_t)kKB * dh, 0.f);
-            s.qv.assign((size_t)G * kQB * dh, 0.f);
-            s.ov.assign((size_t)G * kQB * dh, 0.f);
+            const int qcols = (G * kQB + kNR - 1) / kNR * kNR;
+            const int dpan = (dh + kMR - 1) / kMR, kpan = (kKB + kMR - 1) / kMR;
+            s.qpk.assign((size_t)qcols * dh, 0.f);
+            s.kpk.assign((size_t)kpan * dh * kMR, 0.f);
+            s.vpk.assign((size_t)dpan * kKB * kMR, 0.f);
+            s.ppk.assign((size_t)qcols * kKB, 0.f);
+            s.st.assign((size_t)qcols * kKB, 0.f);
+            s.ot.assign((size_t)qcols * dh, 0.f);
             s.mx.assign((size_t)G * kQB, 0.f);
             s.l.assign((size_t)G * kQB, 0.f);
-            s.s.assign(kKB, 0.f);
         }
         // rotary table in double: angle pos * base^(-2j/dh)
         m->rope.resize((size_t)T * dh);
@@ -587,6 +640,7 @@ vla_status vla_cpu_model_create(const vla_config* cfg, const vla_layer_weights* 
         m->xmid.resize((size_t)T * D);
         m->mbuf.resize((size_t)T * m->F_pad);
         m->rinv.resize(T);
+        m->xrows.resize((size_t)kGemvRows * std::max(std::max(D, m->qc), m->F_pad));
     } catch (const std::bad_alloc&) {
         delete m;
         return VLA_ERR_OOM;

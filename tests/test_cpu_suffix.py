@@ -162,7 +162,8 @@ def test_partition_identity_in_place_and_thread_count(vla):
 
 def test_causal_invariance_and_chunked_prefill(vla):
     """Rows of a prefix of the frame do not depend on later tokens, and a frame prefilled in
-    two calls (the second at p0 = first call's length) equals one call, bit for bit."""
+    chunks (each at p0 = the previous chunks' length) equals one call, bit for bit, also
+    through the weight-streaming path of calls of at most 4 tokens (decode steps)."""
     s, L, M, M1, max_ctx = synth.TINY, 2, 64, 37, 64
     m = CpuModel(vla, s, L, 8, max_ctx, n_threads=4)
     try:
@@ -175,6 +176,10 @@ def test_causal_invariance_and_chunked_prefill(vla):
         np.testing.assert_array_equal(y1, y[:M1])
         y2 = m.run(xb[M1:].copy(), 0, L, kv)
         np.testing.assert_array_equal(y2, y[M1:])
+        vla.vla_cpu_kv_reset(kv)
+        m.run(xb[:M1].copy(), 0, L, kv)
+        for a, b in ((M1, M1 + 3), (M1 + 3, M1 + 4), (M1 + 4, M)):
+            np.testing.assert_array_equal(m.run(xb[a:b].copy(), 0, L, kv), y[a:b])
         vla.vla_cpu_kv_destroy(kv)
     finally:
         m.close()
