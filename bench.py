@@ -39,6 +39,7 @@ PIPELINE_WORKLOAD = "7b_pipeline32_3072tok"
 BLOCK_WORKLOAD = "7b_block_1024tok"
 PIPELINE_SPLITS = (8, 16, 24)
 HYBRID_SPLIT = 31  # GPU blocks [0, 31), the last block on the host cores
+HYBRID_ZONE_MIN = 28  # dynamic zone [28, 32] of the scheduled run
 
 
 def _peaks():
@@ -248,34 +249,53 @@ def _dec_gateup(dstages: dict, s, D: int) -> dict | None:
             "timing": "stage-timed pass: plain launches, without the graph's programmatic overlap"}
 
 
-def hybrid_pipeline(vla, p, s, pwl, xs, stream, seed: int, k: int, torch) -> dict:
+def _pipeline_frames(vla, pl, xs, Mp, D, stream, choose_split, on_done=None) -> list:
+    """Submits every frame as soon as a ring slot is free (split from choose_split(backlog)),
+    collects them in order; returns each frame's stage times."""
+    res, f = [], 0
+    while len(res) < len(xs):
+        while f < len(xs):
+            try:
+                vla.vla_pipeline_submit(pl, f, xs[f], Mp, choose_split(f - len(res)), stream)
+            except vla.VlaError as e:
+                if e.name != "VLA_ERR_BUSY":
+                    raise
+                break
+            f += 1
+        out = np.empty((Mp, D), dtype=np.uint16)
+        fid, t = vla.vla_pipeline_collect(pl, out, 600000)
+        assert fid == len(res)
+        if on_done:
+            on_done(t)
+        res.append(t.as_dict())
+    return res
+
+
+def hybrid_pipeline(vla, p, s, pwl, xs, stream, seed: int, k: int, zone_min: int, torch) -> dict:
     """Frames of the pipeline workload through vla_pipeline (GPU blocks [0, k), CPU blocks
-    [k, N)); per-frame T_G, T_X, T_C (Eq. 12-14) and the steady interval between frames."""
+    [k, N)); per-frame T_G, T_X, T_C (Eq. 8-10) and the steady interval between frames (Eq. 13).
+    Then the same frames with the split chosen per frame by the scheduler (Sec. IV-D) over the
+    dynamic zone [zone_min, N], starting from zone_min + 2."""
     D, N, Mp = s.hidden, pwl.n_layers, pwl.n_tokens
     threads = cpu_threads()
     t0 = time.perf_counter()
     cfg = vla.VlaConfig(hidden=D, n_heads=s.n_heads, n_kv_heads=s.n_kv_heads, head_dim=s.head_dim, ffn=s.ffn,
                         rms_eps=s.rms_eps, rope_base=s.rope_base, max_ctx=Mp)
-    cpu = vla.vla_cpu_model_create(cfg, [synth.layer_weights(s, seed, l) for l in range(k, N)], k, threads)
+    cpu = vla.vla_cpu_model_create(cfg, [synth.layer_weights(s, seed, l) for l in range(zone_min, N)], zone_min,
+                                   threads)
     t_create = time.perf_counter() - t0
     pl = vla.vla_pipeline_create(p, cpu, Mp, 2)
-    res = []
+    sched = vla.vla_scheduler_create(N, zone_min, N, zone_min + 2, max_step=1, alpha=0.5)
     try:
-        f = 0
-        while len(res) < len(xs):
-            while f < len(xs):
-                try:
-                    vla.vla_pipeline_submit(pl, f, xs[f], Mp, k, stream)
-                except vla.VlaError as e:
-                    if e.name != "VLA_ERR_BUSY":
-                        raise
-                    break
-                f += 1
-            out = np.empty((Mp, D), dtype=np.uint16)
-            fid, t = vla.vla_pipeline_collect(pl, out, 600000)
-            assert fid == len(res)
-            res.append(t.as_dict())
+        res = _pipeline_frames(vla, pl, xs, Mp, D, stream, lambda backlog: k)
+        def choose(backlog):
+            return vla.vla_scheduler_next(sched, backlog=backlog)
+
+        sres = _pipeline_frames(vla, pl, xs + xs, Mp, D, stream, choose,
+                                on_done=lambda t: vla.vla_scheduler_observe(sched, t))
+        est = vla.vla_scheduler_estimates(sched)
     finally:
+        vla.vla_scheduler_destroy(sched)
         vla.vla_pipeline_destroy(pl)
         vla.vla_cpu_model_destroy(cpu)
     tg = statistics.median(r["t_gpu_ms"] for r in res)
@@ -286,14 +306,20 @@ def hybrid_pipeline(vla, p, s, pwl, xs, stream, seed: int, k: int, torch) -> dic
     waits = [(r["t_ready_s"] - r["t_start_s"]) * 1e3 for r in res[1:]]
     block_flops = 2.0 * Mp * (s.n_heads * s.head_dim * D + 2 * s.n_kv_heads * s.head_dim * D +
                               D * s.n_heads * s.head_dim + 3 * s.ffn * D) + 2.0 * Mp * Mp * s.head_dim * s.n_heads
+    sdone = [r["t_done_s"] for r in sres]
     return {"split": k, "gpu_blocks": k, "cpu_blocks": N - k, "frames": len(res), "tokens": Mp,
             "t_gpu_ms": tg, "t_xfer_ms": tx, "t_cpu_ms": tc,
-            "steady_interval_ms": interval, "eq14_max_ms": max(tg, tx + tc), "eq12_serial_ms": tg + tx + tc,
+            "steady_interval_ms": interval, "eq13_max_ms": max(tg, tx + tc), "eq12_serial_ms": tg + tx + tc,
             "cpu_wait_for_gpu_ms": waits,
             "cpu_suffix_gflops": block_flops * (N - k) / (tc * 1e-3) / 1e9, "cpu_threads": threads,
             "cpu_model_create_s": t_create,
             "note": "depth-2 ring; interval = median gap between consecutive frame completions after the "
-                    "first two; the CPU suffix is the library's C++ block on the host cores"}
+                    "first two; the CPU suffix is the library's C++ block on the host cores",
+            "scheduled": {"zone": [zone_min, N], "splits": [r["split"] for r in sres],
+                          "interval_ms": [round((b - a) * 1e3, 3) for a, b in zip(sdone, sdone[1:])],
+                          "est_ms_per_block": {"gpu": est[0], "cpu": est[1], "xfer_ms": est[2]},
+                          "note": "split chosen per frame by the scheduler from observed stage times "
+                                  "(at most one block per frame), no co-tenant load"}}
 
 
 def run_ours(args, dist: Dist):
@@ -646,7 +672,7 @@ def run_ours(args, dist: Dist):
         # ---- hybrid pipeline (Sec. IV-C, Eq. 12-14): GPU prefix [0, k) of frame t+1 while the
         # host cores run the suffix [k, 32) of frame t, frames handed over in order
         if not args.no_hybrid:
-            pipeline["hybrid"] = hybrid_pipeline(vla, p, s, pwl, xs, main, seed, HYBRID_SPLIT, torch)
+            pipeline["hybrid"] = hybrid_pipeline(vla, p, s, pwl, xs, main, seed, HYBRID_SPLIT, HYBRID_ZONE_MIN, torch)
     clock_info = clocks.stop()
 
     # ---- CPU oracle baseline (rank 0, N = 1 only): 1 block over the whole 2304-token frame

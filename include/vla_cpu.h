@@ -73,7 +73,7 @@ vla_status vla_cpu_kv_data(const vla_cpu_kv* kv, int layer, void** k_plane, void
 vla_status vla_cpu_prefill(vla_cpu_model* m, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
                            vla_cpu_kv* kv, void* hidden_out);
 
-/* Per-frame stage times of the pipeline, the terms of Eq. 12-14:
+/* Per-frame stage times of the pipeline, the stage terms of Eq. 8-10:
  *   t_gpu_ms   T_G: prefix [0, p) on the GPU (CUDA events around it on the submit stream)
  *   t_xfer_ms  T_X: from the end of the prefix to the end of the boundary copy into pinned
  *              host memory (CUDA events; includes waiting for the side stream)
@@ -135,6 +135,50 @@ int vla_pipeline_in_flight(const vla_pipeline* pl);
 /* Waits for the worker to finish the queued frames, joins it and frees everything the
  * pipeline owns (not the models). NULL is a no-op. */
 vla_status vla_pipeline_destroy(vla_pipeline* pl);
+
+/* Flexible resource scheduling (Sec. IV-D, Eq. 15-17). The blocks form a GPU-fixed zone
+ * [0, k_min), a dynamic zone and a CPU-fixed zone [k_max, N); the split p of each frame is one
+ * of the candidate policies {k_min, ..., k_max} (Eq. 16), chosen by a controller Phi from the
+ * runtime state z_t = [u_gpu, u_cpu, q_t] (Eq. 15, 17). The paper does not give Phi; this one:
+ *   - keeps per-block cost estimates, g (GPU) and c (CPU) in ms per block, as exponential
+ *     moving averages of T_G / p and T_C / (N - p) over observed frames, and the transfer
+ *     time x likewise (vla_scheduler_observe; a side with no blocks in a frame is not updated);
+ *   - scales them by the share of each processor other work leaves free: g / (1 - u_gpu),
+ *     c / (1 - u_cpu), with the utilisations clamped to [0, 0.95];
+ *   - predicts the steady interval of Eq. 13, max(p g', x + (N - p) c'), for every candidate
+ *     and moves the split toward the best one (ties: the one nearest the current split) by at
+ *     most max_step blocks per frame, so only boundary-adjacent blocks migrate;
+ *   - when the backlog q_t reaches backlog_limit frames and the prediction asks for no move,
+ *     moves one block away from the stage predicted to be slower;
+ *   - keeps the split while either cost has never been observed. */
+typedef struct {
+    int n_layers;       /* N */
+    int k_min, k_max;   /* 0 <= k_min <= k_max <= N */
+    int k_init;         /* first split, in [k_min, k_max] */
+    int max_step;       /* >= 1 */
+    double alpha;       /* (0, 1]: weight of the newest frame in the moving averages */
+    int backlog_limit;  /* >= 1 */
+} vla_sched_config;
+
+typedef struct {
+    double u_gpu;  /* share of the GPU taken by other work, [0, 1] */
+    double u_cpu;  /* share of the host cores taken by other work, [0, 1] */
+    int backlog;   /* q_t: frames submitted and not yet finished */
+} vla_sched_state;
+
+typedef struct vla_scheduler vla_scheduler;
+
+/* Errors: INVALID_ARG (null or inconsistent config), OOM. */
+vla_status vla_scheduler_create(const vla_sched_config* cfg, vla_scheduler** out);
+/* Folds one finished frame's stage times into the cost estimates. Errors: INVALID_ARG. */
+vla_status vla_scheduler_observe(vla_scheduler* s, const vla_frame_times* t);
+/* Phi(z_t): the split for the next frame (and the scheduler's new current split); -1 if an
+ * argument is NULL. */
+int vla_scheduler_next(vla_scheduler* s, const vla_sched_state* z);
+/* Current estimates (ms per GPU block, ms per CPU block, ms per transfer); a never-observed
+ * one reads -1. Any output may be NULL. Errors: INVALID_ARG. */
+vla_status vla_scheduler_estimates(const vla_scheduler* s, double* g_ms, double* c_ms, double* x_ms);
+vla_status vla_scheduler_destroy(vla_scheduler* s);
 
 #ifdef __cplusplus
 }

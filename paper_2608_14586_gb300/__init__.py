@@ -25,7 +25,8 @@ __all__ = [
     "VlaFrameTimes", "vla_cpu_model_create", "vla_cpu_model_destroy", "vla_cpu_model_threads", "vla_cpu_model_info",
     "vla_cpu_kv_create", "vla_cpu_kv_destroy", "vla_cpu_kv_reset", "vla_cpu_kv_length", "vla_cpu_kv_data",
     "vla_cpu_prefill", "vla_pipeline_create", "vla_pipeline_submit", "vla_pipeline_collect",
-    "vla_pipeline_in_flight", "vla_pipeline_destroy",
+    "vla_pipeline_in_flight", "vla_pipeline_destroy", "VlaSchedConfig", "VlaSchedState", "vla_scheduler_create",
+    "vla_scheduler_observe", "vla_scheduler_next", "vla_scheduler_estimates", "vla_scheduler_destroy",
 ]
 
 # stage ids of vla_prefix_stage_times (VLA_STAGE_* in vla_prefix.h)
@@ -58,7 +59,7 @@ class VlaLayerWeights(ctypes.Structure):
 
 
 class VlaFrameTimes(ctypes.Structure):
-    """Per-frame stage times of the pipeline (vla_frame_times): T_G, T_X, T_C of Eq. 12-14."""
+    """Per-frame stage times of the pipeline (vla_frame_times): T_G, T_X, T_C of Eq. 8-10."""
     _fields_ = [("t_gpu_ms", ctypes.c_double), ("t_xfer_ms", ctypes.c_double), ("t_cpu_ms", ctypes.c_double),
                 ("t_submit_s", ctypes.c_double), ("t_start_s", ctypes.c_double), ("t_ready_s", ctypes.c_double),
                 ("t_done_s", ctypes.c_double),
@@ -66,6 +67,18 @@ class VlaFrameTimes(ctypes.Structure):
 
     def as_dict(self) -> dict:
         return {n: getattr(self, n) for n, _ in self._fields_}
+
+
+class VlaSchedConfig(ctypes.Structure):
+    """Zones and controller settings of the split scheduler (vla_sched_config)."""
+    _fields_ = [("n_layers", ctypes.c_int), ("k_min", ctypes.c_int), ("k_max", ctypes.c_int),
+                ("k_init", ctypes.c_int), ("max_step", ctypes.c_int), ("alpha", ctypes.c_double),
+                ("backlog_limit", ctypes.c_int)]
+
+
+class VlaSchedState(ctypes.Structure):
+    """Runtime state z_t = [u_gpu, u_cpu, q_t] of Eq. 15 (vla_sched_state)."""
+    _fields_ = [("u_gpu", ctypes.c_double), ("u_cpu", ctypes.c_double), ("backlog", ctypes.c_int)]
 
 
 _lib = None
@@ -127,6 +140,12 @@ def load():
         "vla_pipeline_collect": ([P, ctypes.POINTER(ctypes.c_int64), V, I, ctypes.POINTER(VlaFrameTimes)], I),
         "vla_pipeline_in_flight": ([P], I),
         "vla_pipeline_destroy": ([P], I),
+        "vla_scheduler_create": ([ctypes.POINTER(VlaSchedConfig), ctypes.POINTER(P)], I),
+        "vla_scheduler_observe": ([P, ctypes.POINTER(VlaFrameTimes)], I),
+        "vla_scheduler_next": ([P, ctypes.POINTER(VlaSchedState)], I),
+        "vla_scheduler_estimates": ([P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double),
+                                     ctypes.POINTER(ctypes.c_double)], I),
+        "vla_scheduler_destroy": ([P], I),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -415,3 +434,34 @@ def vla_pipeline_in_flight(pl) -> int:
 
 def vla_pipeline_destroy(pl):
     _check(load().vla_pipeline_destroy(pl), "vla_pipeline_destroy")
+
+
+def vla_scheduler_create(n_layers: int, k_min: int, k_max: int, k_init: int, max_step: int = 1,
+                         alpha: float = 0.5, backlog_limit: int = 2) -> ctypes.c_void_p:
+    """Split-point controller Phi over the dynamic zone [k_min, k_max] (Sec. IV-D)."""
+    cfg = VlaSchedConfig(n_layers=n_layers, k_min=k_min, k_max=k_max, k_init=k_init, max_step=max_step,
+                         alpha=alpha, backlog_limit=backlog_limit)
+    out = ctypes.c_void_p()
+    _check(load().vla_scheduler_create(ctypes.byref(cfg), ctypes.byref(out)), "vla_scheduler_create")
+    return out
+
+
+def vla_scheduler_observe(s, times: VlaFrameTimes):
+    _check(load().vla_scheduler_observe(s, ctypes.byref(times)), "vla_scheduler_observe")
+
+
+def vla_scheduler_next(s, u_gpu: float = 0.0, u_cpu: float = 0.0, backlog: int = 0) -> int:
+    z = VlaSchedState(u_gpu=u_gpu, u_cpu=u_cpu, backlog=backlog)
+    return load().vla_scheduler_next(s, ctypes.byref(z))
+
+
+def vla_scheduler_estimates(s) -> tuple:
+    """(ms per GPU block, ms per CPU block, ms per transfer); -1 where never observed."""
+    g, c, x = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    _check(load().vla_scheduler_estimates(s, ctypes.byref(g), ctypes.byref(c), ctypes.byref(x)),
+           "vla_scheduler_estimates")
+    return g.value, c.value, x.value
+
+
+def vla_scheduler_destroy(s):
+    _check(load().vla_scheduler_destroy(s), "vla_scheduler_destroy")
