@@ -4,9 +4,10 @@
 // once from HBM (354 MB per 7B-class block), so these kernels are built for bandwidth:
 //   * one warp per pair of weight rows, 16-byte non-allocating loads, 8 chunks per row in
 //     flight per lane, fp32 FMA, warp-shuffle reduction;
-//   * the pair is chosen so the fused epilogue has both operands it needs: rows (j, j+dh/2)
-//     of a head for the rotary embedding, the gate and up rows of one feed-forward unit for
-//     SwiGLU, consecutive rows for the residual projections;
+//   * the pair is chosen so the fused epilogue has both operands it needs: dims (j, j+dh/2)
+//     of a head for the rotary embedding (adjacent rows of the repacked q/k weights), the
+//     gate and up rows of one feed-forward unit for SwiGLU, consecutive rows for the
+//     residual projections;
 //   * the input vector is staged in shared memory; RMSNorm's 1/rms is computed per CTA
 //     (the gains are folded into the weights);
 //   * under programmatic dependent launch each kernel starts while its predecessor drains:
@@ -68,8 +69,13 @@ VLA_DEV void unit_rows(const GemvParams& p, int u, int& ra, int& rb) {
     if constexpr (MODE == kGemvQKV) {
         const int half = p.dh >> 1;
         const int head = u / half, j = u % half;
-        ra = head * p.dh + j;
-        rb = ra + half;
+        if (head < p.n_q_heads + p.n_kv_heads) {  // q, k: the pair's rows are adjacent
+            ra = head * p.dh + 2 * j;
+            rb = ra + 1;
+        } else {
+            ra = head * p.dh + j;
+            rb = ra + half;
+        }
     } else if constexpr (MODE == kGemvSwiGLU) {
         const int grp = u >> 7, i = u & 127;
         ra = grp * 256 + i;

@@ -77,8 +77,10 @@ __global__ void repack_kernel(RepackSrc s, RepackDst d, int D, int H, int Hkv, i
             const int k = (int)(j % D);
             const float gk = __bfloat162float(s.g_attn[k]);
             float w;
-            if (r < qn) w = __bfloat162float(s.w_q[r * D + k]);
-            else if (r < qn + kvn) w = __bfloat162float(s.w_k[(r - qn) * D + k]);
+            // q and k heads: row 2j + e holds source row j + e * dh/2 (rotation pairs adjacent)
+            const long long rs = (r < qn + kvn) ? (r / dh) * dh + ((r % dh) >> 1) + ((r % dh) & 1) * (dh >> 1) : r;
+            if (r < qn) w = __bfloat162float(s.w_q[rs * D + k]);
+            else if (r < qn + kvn) w = __bfloat162float(s.w_k[(rs - qn) * D + k]);
             else w = __bfloat162float(s.w_v[(r - qn - kvn) * D + k]);
             d.w_qkv[j] = __float2bfloat16_rn(w * gk);
             continue;

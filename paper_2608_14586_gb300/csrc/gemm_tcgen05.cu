@@ -14,8 +14,10 @@
 // Tiles are walked M-fastest so CTAs running together share the weight (B) tiles in L2.
 //
 // Fused epilogues (the block stages of the decoder, see the header of runtime.cu):
-//   kEpiQKV     RMSNorm row scale, rotate-half RoPE of q and k, q to the query buffer,
-//               post-RoPE k and v to the layer's KV cache at positions pos0 + row
+//   kEpiQKV     RMSNorm row scale, rotate-half RoPE of q and k (the weights hold each rotation
+//               pair in adjacent rows, so any 32-column chunk is whole pairs and tiles of 192
+//               columns are possible), q to the query buffer, post-RoPE k and v to the layer's
+//               KV cache at positions pos0 + row
 //   kEpiResid   residual add (attention output projection, MLP down projection)
 //   kEpiSwiGLU  RMSNorm row scale and silu(gate) * up on 128-column interleaved tiles
 #include "common.cuh"
@@ -31,11 +33,11 @@ constexpr int kThreads = 192;
 
 template <int BN>
 struct GemmCfg {
-    static constexpr int STAGES = (BN == 256) ? 4 : 6;
+    static constexpr int STAGES = (BN == 256) ? 4 : (BN == 192 ? 5 : 6);
     static constexpr uint32_t A_BYTES = kBM * kBK * 2;
     static constexpr uint32_t B_BYTES = BN * kBK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr uint32_t TMEM_COLS = 2 * BN;
+    static constexpr uint32_t TMEM_COLS = (BN == 192) ? 512 : 2 * BN;  // a power of two
     static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
 };
@@ -140,6 +142,23 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
     if (ep.ss_out && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_chunks + n0 / 256] = ss;
 }
 
+VLA_DEV void store_bf16x16(bf16* dst, const float* v) {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        uint4 o;
+        o.x = pack_bf16x2(v[i * 8 + 0], v[i * 8 + 1]);
+        o.y = pack_bf16x2(v[i * 8 + 2], v[i * 8 + 3]);
+        o.z = pack_bf16x2(v[i * 8 + 4], v[i * 8 + 5]);
+        o.w = pack_bf16x2(v[i * 8 + 6], v[i * 8 + 7]);
+        d[i] = o;
+    }
+}
+
+// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
+// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
+// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
+// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order.
 template <int BN>
 VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const bool row_ok = row < ep.M;
@@ -147,55 +166,40 @@ VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const int pos = ep.pos0 + row;
     const int dh = ep.head_dim;
     const int half = dh >> 1;
-    const int region = (n0 < ep.q_cols) ? 0 : ((n0 < ep.q_cols + ep.kv_cols) ? 1 : 2);
-    if (region == 2) {
-        // values: no rotation
+    const float2* rope = ep.rope + (size_t)(row_ok ? pos : 0) * half;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
-            uint32_t r[32];
-            tmem_ld32(taddr + c, r);
-            if (!row_ok) continue;
-            const int n = n0 + c - ep.q_cols - ep.kv_cols;
+    for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        const int col = n0 + c;
+        if (!row_ok || col >= ep.N) continue;
+        if (col >= ep.q_cols + ep.kv_cols) {
+            const int n = col - ep.q_cols - ep.kv_cols;
             const int g = n / dh, d = n % dh;
             float v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = f32(r[i]) * s;
             store_bf16x32(ep.vcache + ((size_t)g * ep.max_ctx + pos) * dh + d, v);
+            continue;
         }
-        return;
-    }
-    const float2* rope = ep.rope + (size_t)(row_ok ? pos : 0) * half;
-#pragma unroll 1
-    for (int hb = 0; hb < BN; hb += dh) {
-#pragma unroll 1
-        for (int c = 0; c < half; c += 32) {
-            uint32_t ra[32], rb[32];
-            tmem_ld32(taddr + hb + c, ra);
-            tmem_ld32(taddr + hb + half + c, rb);
-            if (!row_ok) continue;
-            float va[32], vb[32];
+        const bool is_q = col < ep.q_cols;
+        const int n = is_q ? col : col - ep.q_cols;
+        const int head = n / dh, i0 = (n % dh) >> 1;
+        float va[16], vb[16];
 #pragma unroll
-            for (int i = 0; i < 32; i += 2) {  // 16-byte loads: two (cos, sin) pairs each
-                const float4 cs = __ldg(reinterpret_cast<const float4*>(rope + c + i));
-                const float a0 = f32(ra[i]) * s, b0 = f32(rb[i]) * s;
-                const float a1 = f32(ra[i + 1]) * s, b1 = f32(rb[i + 1]) * s;
-                va[i] = a0 * cs.x - b0 * cs.y;
-                vb[i] = b0 * cs.x + a0 * cs.y;
-                va[i + 1] = a1 * cs.z - b1 * cs.w;
-                vb[i + 1] = b1 * cs.z + a1 * cs.w;
-            }
-            if (region == 0) {
-                bf16* op = ep.out + (size_t)row * ep.ld_out + n0 + hb + c;
-                store_bf16x32(op, va);
-                store_bf16x32(op + half, vb);
-            } else {
-                const int n = n0 + hb - ep.q_cols;
-                const int g = n / dh;
-                bf16* kp = ep.kcache + ((size_t)g * ep.max_ctx + pos) * dh + c;
-                store_bf16x32(kp, va);
-                store_bf16x32(kp + half, vb);
-            }
+        for (int i = 0; i < 16; i += 2) {  // 16-byte loads: two (cos, sin) pairs each
+            const float4 cs = __ldg(reinterpret_cast<const float4*>(rope + i0 + i));
+            const float a0 = f32(r[2 * i]) * s, b0 = f32(r[2 * i + 1]) * s;
+            const float a1 = f32(r[2 * i + 2]) * s, b1 = f32(r[2 * i + 3]) * s;
+            va[i] = a0 * cs.x - b0 * cs.y;
+            vb[i] = b0 * cs.x + a0 * cs.y;
+            va[i + 1] = a1 * cs.z - b1 * cs.w;
+            vb[i + 1] = b1 * cs.z + a1 * cs.w;
         }
+        bf16* dst = is_q ? ep.out + (size_t)row * ep.ld_out + (size_t)head * dh
+                         : ep.kcache + ((size_t)head * ep.max_ctx + pos) * dh;
+        store_bf16x16(dst + i0, va);
+        store_bf16x16(dst + i0 + half, vb);
     }
 }
 
@@ -457,13 +461,15 @@ cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMa
             case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
             case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream, pdl);
         }
+    } else if (bn == 192) {
+        if (mode == kEpiQKV) return launch_one<192, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
     } else if (bn == 128) {
         switch (mode) {
             case kEpiPlain:
             case kEpiResid:
                 if (ep.ss_out) return cudaErrorInvalidValue;  // row partials are per 256 columns
                 return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
-            case kEpiQKV: return launch_one<128, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiQKV: return cudaErrorInvalidValue;  // BN = 256 or 192 only
             case kEpiSwiGLU: return cudaErrorInvalidValue;  // gate/up rows are interleaved for BN = 256
         }
     }

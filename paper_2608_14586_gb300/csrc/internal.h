@@ -100,7 +100,8 @@ struct RepackSrc {
     const bf16 *w_q, *w_k, *w_v, *w_o, *w_gate, *w_up, *w_down, *g_attn, *g_mlp;
 };
 struct RepackDst {
-    bf16* w_qkv;  // [H*dh + 2*Hkv*dh, D], rows of q | k | v, each column scaled by g_attn
+    bf16* w_qkv;  // [H*dh + 2*Hkv*dh, D], rows of q | k | v, each column scaled by g_attn; within
+                  // each q and k head the rotation pairs (j, j + dh/2) sit in rows (2j, 2j + 1)
     bf16* w_o;    // [D, H*dh]
     bf16* w_gu;   // [2*F_pad, D], 256-row groups = 128 gate rows then 128 up rows, scaled by g_mlp
     bf16* w_d;    // [D, F_pad], columns >= F zero

@@ -106,7 +106,7 @@ constexpr int kMaxDecodeGraphs = 8;
 
 struct LayerDev {
     bf16 *w_qkv, *w_o, *w_gu, *w_d;
-    CUtensorMap tm_qkv, tm_o, tm_gu, tm_d;
+    CUtensorMap tm_qkv, tm_qkv192, tm_o, tm_gu, tm_d;  // tm_qkv192: 192-row boxes of W_qkv
 };
 
 }  // namespace
@@ -341,6 +341,7 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         e = vla::launch_repack(s, d, D, H, Hkv, dh, cfg->ffn, p->F_pad, 0);
         if (e != cudaSuccess) break;
         if (!vla::make_tmap_bf16(&ld.tm_qkv, ld.w_qkv, p->qkv_n, D, D, kBN) ||
+            !vla::make_tmap_bf16(&ld.tm_qkv192, ld.w_qkv, p->qkv_n, D, D, 192) ||
             !vla::make_tmap_bf16(&ld.tm_o, ld.w_o, D, p->qc, p->qc, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_gu, ld.w_gu, 2 * p->F_pad, D, D, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_d, ld.w_d, D, p->F_pad, p->F_pad, kBN)) {
@@ -500,6 +501,14 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         first_launch = false;
         return r;
     };
+    // QKV tile width: the one with fewer column-slots in its last wave of tiles (waves x width;
+    // 192 pays where 256-wide tiles leave a mostly idle second wave, e.g. 1024 tokens of a 7B
+    // block: 192 tiles of 256 on 152 SMs, 256 tiles of 192), 256 on a tie
+    auto wave_cost = [&](int bn) {
+        const long long tiles = (long long)((M + 127) / 128) * ((p->qkv_n + bn - 1) / bn);
+        return ((tiles + p->num_sms - 1) / p->num_sms) * bn;
+    };
+    const int qkv_bn = wave_cost(192) < wave_cost(kBN) ? 192 : kBN;
     for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
         const LayerDev& ld = p->layers[l];
         const bf16* x = (l == layer_begin) ? (const bf16*)hidden_in : (const bf16*)hidden_out;
@@ -534,8 +543,8 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ep.len_value = p0 + M;
         ep.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_QKV, true);
-        e = vla::launch_gemm(vla::kEpiQKV, kBN, tm_x, ld.tm_qkv, M, p->qkv_n, D, ep, p->num_sms, stream,
-                             pdl(VLA_STAGE_GEMM_QKV));
+        e = vla::launch_gemm(vla::kEpiQKV, qkv_bn, tm_x, qkv_bn == 192 ? ld.tm_qkv192 : ld.tm_qkv, M, p->qkv_n, D,
+                             ep, p->num_sms, stream, pdl(VLA_STAGE_GEMM_QKV));
         stage_mark(p, VLA_STAGE_GEMM_QKV, false);
         if (e != cudaSuccess) break;
         // causal GQA attention over the cache
