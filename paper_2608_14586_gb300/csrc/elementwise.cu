@@ -7,21 +7,23 @@ namespace vla {
 
 namespace {
 
-// Row sums of squares per 256-column chunk, in exactly the order the residual GEMM epilogue
-// forms them for its stored outputs: each 32-column group is an fp32 fmaf chain from zero over
-// its columns in order, and the chunk's sum adds the 8 group values in order. One thread per
-// group; the 8 threads of a chunk are consecutive lanes.
-__global__ void row_sumsq_kernel(const bf16* __restrict__ x, int M, int chunks, int ld, float* __restrict__ ss) {
+// Row sums of squares in exactly the order the residual GEMM epilogue forms them for its
+// stored outputs: per 32-column group an fp32 fmaf chain from zero over its columns in order;
+// for WIDTH 256 the 8 group sums of a chunk are then added in group order. One thread per
+// 32-column group; with WIDTH 256 the 8 threads of a chunk are consecutive lanes.
+template <int WIDTH>
+__global__ void row_sumsq_kernel(const bf16* __restrict__ x, int M, int groups, int ld, float* __restrict__ ss) {
+    constexpr int SUB = WIDTH / 32;  // 32-column groups per partial
     const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     pdl_wait();  // x is the previous kernel's output
     pdl_trigger();
-    const long long chunk = i >> 3;
-    const int grp = (int)(i & 7);
-    const bool ok = chunk < (long long)M * chunks;
+    const long long part = i / SUB;
+    const int sub = (int)(i % SUB);
+    const bool ok = part < (long long)M * groups;
     float g = 0.f;
     if (ok) {
-        const int row = (int)(chunk / chunks), t = (int)(chunk % chunks);
-        const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * ld + t * 256 + grp * 32);
+        const int row = (int)(part / groups), t = (int)(part % groups);
+        const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)row * ld + t * WIDTH + sub * 32);
         uint4 v[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) v[c] = xr[c];
@@ -36,16 +38,20 @@ __global__ void row_sumsq_kernel(const bf16* __restrict__ x, int M, int chunks, 
             }
         }
     }
-    // the chunk's 8 group sums to its first lane, added in group order
-    const int base = threadIdx.x & 24;  // first lane of this octet
-    float part[8];
+    if constexpr (SUB == 1) {
+        if (ok) ss[part] = g;
+    } else {
+        // the chunk's group sums to its first lane, added in group order
+        const int base = threadIdx.x & (32 - SUB);
+        float sums[SUB];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) part[k] = __shfl_sync(0xFFFFFFFFu, g, base + k);
-    if (ok && grp == 0) {
-        float t = 0.f;
+        for (int k = 0; k < SUB; ++k) sums[k] = __shfl_sync(0xFFFFFFFFu, g, base + k);
+        if (ok && sub == 0) {
+            float t = 0.f;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) t += part[k];
-        ss[chunk] = t;
+            for (int k = 0; k < SUB; ++k) t += sums[k];
+            ss[part] = t;
+        }
     }
 }
 
@@ -117,12 +123,15 @@ __global__ void set_lengths_kernel(int* d_len, int count, int value) {
 
 }  // namespace
 
-cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl) {
+cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, int width, float* ss, cudaStream_t stream,
+                             bool pdl) {
     if (M <= 0) return cudaSuccess;
-    const int chunks = D / 256;
-    const long long n = (long long)M * chunks * 8;  // one thread per 32-column group
-    return launch_ex(row_sumsq_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, stream, pdl, x, M, chunks, ld,
-                     ss);
+    const int groups = D / width;
+    const long long n = (long long)M * (D / 32);  // one thread per 32-column group
+    const dim3 grid((unsigned)((n + 255) / 256));
+    if (width == 256) return launch_ex(row_sumsq_kernel<256>, grid, dim3(256), 0, stream, pdl, x, M, groups, ld, ss);
+    if (width == 32) return launch_ex(row_sumsq_kernel<32>, grid, dim3(256), 0, stream, pdl, x, M, groups, ld, ss);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream) {

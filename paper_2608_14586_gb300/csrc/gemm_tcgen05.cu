@@ -33,11 +33,12 @@ constexpr int kThreads = 192;
 
 template <int BN>
 struct GemmCfg {
-    static constexpr int STAGES = (BN == 256) ? 4 : (BN == 192 ? 5 : 6);
     static constexpr uint32_t A_BYTES = kBM * kBK * 2;
     static constexpr uint32_t B_BYTES = BN * kBK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr uint32_t TMEM_COLS = (BN == 192) ? 512 : 2 * BN;  // a power of two
+    // as many stages as fit in 227 KB next to the alignment pad and barriers, at most 6
+    static constexpr int STAGES = (232448 - 1280) / STAGE_BYTES < 6 ? (232448 - 1280) / STAGE_BYTES : 6;
+    static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;  // two accumulators, a power of two
     static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
 };
@@ -61,26 +62,30 @@ VLA_DEV void store_bf16x32(bf16* dst, const float (&v)[32]) {
 // Epilogues. Each thread owns one output row (TMEM lane); all 32 lanes of a warp execute
 // every tcgen05.ld; stores are masked per row / column.
 // ---------------------------------------------------------------------------------------
-// 1/rms of an input row from its 256-column partial sums of squares (chunk order)
+// 1/rms of an input row from its 32-column partial sums of squares, added in group order
 VLA_DEV float row_rinv(const EpiParams& ep, int row) {
-    const float* ps = ep.ss_in + (size_t)row * ep.ss_chunks;
+    const float* ps = ep.ss_in + (size_t)row * ep.ss_groups;
     float t = 0.f;
-    if ((ep.ss_chunks & 3) == 0 && ep.ss_chunks <= 32) {  // 16-byte loads issued before the in-order sum
-        const int n4 = ep.ss_chunks >> 2;
-        float4 q[8];
+    if ((ep.ss_groups & 3) == 0) {  // batches of eight 16-byte loads, each summed in order
+        const float4* p4 = reinterpret_cast<const float4*>(ps);
+        const int n4 = ep.ss_groups >> 2;
+#pragma unroll 1
+        for (int b = 0; b < n4; b += 8) {
+            float4 q[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) q[i] = i < n4 ? __ldcg(reinterpret_cast<const float4*>(ps) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int i = 0; i < 8; ++i) q[i] = b + i < n4 ? __ldcg(p4 + b + i) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            if (i < n4) {
-                t += q[i].x;
-                t += q[i].y;
-                t += q[i].z;
-                t += q[i].w;
+            for (int i = 0; i < 8; ++i) {
+                if (b + i < n4) {
+                    t += q[i].x;
+                    t += q[i].y;
+                    t += q[i].z;
+                    t += q[i].w;
+                }
             }
         }
     } else {
-        for (int c = 0; c < ep.ss_chunks; ++c) t += ps[c];
+        for (int c = 0; c < ep.ss_groups; ++c) t += ps[c];
     }
     return 1.0f / sqrtf(t / (float)ep.norm_dim + ep.eps);
 }
@@ -88,7 +93,7 @@ VLA_DEV float row_rinv(const EpiParams& ep, int row) {
 template <int BN>
 VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     const bool row_ok = row < ep.M;
-    float ss = 0.f;  // sum of squares of the stored outputs (32-column groups in order)
+    float ss = 0.f;  // ss_width 256: the tile's 256-column partial, its 8 group sums in order
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
         uint32_t r[32];
@@ -117,14 +122,15 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
             }
             store_bf16x32(op, v);
             if (ep.out_host) store_bf16x32(ep.out_host + (size_t)row * ep.ld_out + col, v);
-            if (ep.ss_out) {  // per 32 columns a chain from zero, the groups then added in order
+            if (ep.ss_out) {  // the group's sum of squares of the stored values, a chain from zero
                 float g = 0.f;
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
                     const float r = __bfloat162float(__float2bfloat16_rn(v[i]));
                     g = fmaf(r, r, g);
                 }
-                ss += g;
+                if (ep.ss_width == 32) ep.ss_out[(size_t)row * ep.ss_groups + (col >> 5)] = g;
+                else ss += g;
             }
         } else {
 #pragma unroll
@@ -138,8 +144,7 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
             }
         }
     }
-    // the row statistics of the next RMSNorm (BN = 256: one partial per 256-column chunk)
-    if (ep.ss_out && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_chunks + n0 / 256] = ss;
+    if (ep.ss_out && ep.ss_width == 256 && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_groups + n0 / 256] = ss;
 }
 
 VLA_DEV void store_bf16x16(bf16* dst, const float* v) {
@@ -461,13 +466,16 @@ cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMa
             case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
             case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream, pdl);
         }
+    } else if (bn == 224) {
+        if (ep.ss_out && ep.ss_width != 32) return cudaErrorInvalidValue;  // partials would straddle tiles
+        if (mode == kEpiResid || mode == kEpiPlain) return launch_one<224, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
     } else if (bn == 192) {
         if (mode == kEpiQKV) return launch_one<192, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
     } else if (bn == 128) {
         switch (mode) {
             case kEpiPlain:
             case kEpiResid:
-                if (ep.ss_out) return cudaErrorInvalidValue;  // row partials are per 256 columns
+                if (ep.ss_out && ep.ss_width != 32) return cudaErrorInvalidValue;
                 return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
             case kEpiQKV: return cudaErrorInvalidValue;  // BN = 256 or 192 only
             case kEpiSwiGLU: return cudaErrorInvalidValue;  // gate/up rows are interleaved for BN = 256

@@ -28,13 +28,16 @@ struct EpiParams {
     const bf16* resid;
     int ld_resid;
     // RMSNorm of the GEMM's input rows: 1/rms = 1/sqrt(sum_t ss_in[row][t] / D + eps), the
-    // partial sums of squares over 256-column chunks added in chunk order (kEpiQKV, kEpiSwiGLU)
+    // partial sums of squares of ss_width-column groups added in group order (kEpiQKV,
+    // kEpiSwiGLU). A partial is the in-order sum of its 32-column sub-groups, each an fmaf
+    // chain from zero over its columns in order.
     const float* ss_in;
-    int ss_chunks;  // D / 256
+    int ss_width;   // 256 (tiles of 256 columns) or 32 (any tile width that is a multiple of 32)
+    int ss_groups;  // D / ss_width
     int norm_dim;   // D
     float eps;
-    // kEpiResid: per-row partial sums of squares of the stored (bf16) outputs of this tile's
-    // 256 columns -> ss_out[row][n0 / 256] (nullptr: not wanted)
+    // kEpiResid: the same partials of the stored (bf16) outputs -> ss_out[row][col / ss_width]
+    // (nullptr: not wanted; ss_width 256 needs 256-wide tiles)
     float* ss_out;
     // QKV epilogue
     bf16* kcache;        // layer base, [n_kv_heads][max_ctx][head_dim]
@@ -90,7 +93,10 @@ cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status,
 // over 32-column groups added in group order: the same partial sums the residual GEMM epilogue
 // writes for its output, so a block gets bit-identical row statistics whether its input came
 // from the previous block or from the caller.
-cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, float* ss, cudaStream_t stream, bool pdl = false);
+// ss[row][t] = the row's sum of squares over columns [t*width, (t+1)*width), in the order
+// EpiParams describes (width 256 or 32)
+cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, int width, float* ss, cudaStream_t stream,
+                             bool pdl = false);
 
 // cos/sin table [max_ctx][dh/2] from float64 angles pos * base^(-2j/dh)
 cudaError_t launch_rope_table(float2* table, int max_ctx, int head_dim, double base, cudaStream_t stream);

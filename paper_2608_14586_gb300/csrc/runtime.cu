@@ -1,7 +1,7 @@
 // C-ABI runtime of the LLM-prefix library (include/vla_prefix.h, include/vla_ops.h).
 //
 // Per block l of a prefill over [layer_begin, layer_end), on the caller's stream:
-//   row_sumsq(x)        (first block)  sum of x^2 per 256-column chunk      (RMSNorm statistics)
+//   row_sumsq(x)        (first block)  sum of x^2 per 32-column group       (RMSNorm statistics)
 //   GEMM  x * Wqkv^T   [kEpiQKV]       1/rms scale, RoPE, q -> workspace,   (RMSNorm, projection,
 //                                      post-RoPE k and v -> KV cache         RoPE, KV write)
 //   attention(q, K, V)                 causal GQA over cache [0, p0 + M)
@@ -106,7 +106,8 @@ constexpr int kMaxDecodeGraphs = 8;
 
 struct LayerDev {
     bf16 *w_qkv, *w_o, *w_gu, *w_d;
-    CUtensorMap tm_qkv, tm_qkv192, tm_o, tm_gu, tm_d;  // tm_qkv192: 192-row boxes of W_qkv
+    // tm_qkv192 / tm_o224 / tm_d224: the same weights in 192- and 224-row boxes
+    CUtensorMap tm_qkv, tm_qkv192, tm_o, tm_o224, tm_gu, tm_d, tm_d224;
 };
 
 }  // namespace
@@ -121,7 +122,7 @@ struct vla_prefix {
     float2* rope = nullptr;
     // prefill workspace, sized for cfg.max_ctx tokens
     bf16 *ws_q = nullptr, *ws_attn = nullptr, *ws_xmid = nullptr, *ws_m = nullptr;
-    float *ws_ss_x = nullptr, *ws_ss_mid = nullptr;  // [max_ctx][D/256] row sums of squares
+    float *ws_ss_x = nullptr, *ws_ss_mid = nullptr;  // [max_ctx][D/32] row sums of squares
     // decode workspace
     float* dq = nullptr;
     bf16 *d_attn = nullptr, *d_xmid = nullptr, *d_m = nullptr;
@@ -311,8 +312,8 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
     bool ok = dmalloc(&p->weight_pool, per_layer * layer_count) && dmalloc(&p->rope, (size_t)T * dh / 2) &&
               dmalloc(&p->ws_q, (size_t)T * p->qc) && dmalloc(&p->ws_attn, (size_t)T * p->qc) &&
               dmalloc(&p->ws_xmid, (size_t)T * D) && dmalloc(&p->ws_m, (size_t)T * p->F_pad) &&
-              dmalloc(&p->ws_ss_x, (size_t)T * (D / 256)) &&
-              dmalloc(&p->ws_ss_mid, (size_t)T * (D / 256)) && dmalloc(&p->dq, (size_t)vla::kMaxDecodeBatch * p->qc) &&
+              dmalloc(&p->ws_ss_x, (size_t)T * (D / 32)) &&
+              dmalloc(&p->ws_ss_mid, (size_t)T * (D / 32)) && dmalloc(&p->dq, (size_t)vla::kMaxDecodeBatch * p->qc) &&
               dmalloc(&p->d_attn, (size_t)vla::kMaxDecodeBatch * p->qc) &&
               dmalloc(&p->d_xmid, (size_t)vla::kMaxDecodeBatch * D) &&
               dmalloc(&p->d_m, (size_t)vla::kMaxDecodeBatch * p->F_pad) && dmalloc(&p->d_status, 1) &&
@@ -343,6 +344,8 @@ vla_status vla_prefix_create(const vla_config* cfg, const vla_layer_weights* wei
         if (!vla::make_tmap_bf16(&ld.tm_qkv, ld.w_qkv, p->qkv_n, D, D, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_qkv192, ld.w_qkv, p->qkv_n, D, D, 192) ||
             !vla::make_tmap_bf16(&ld.tm_o, ld.w_o, D, p->qc, p->qc, kBN) ||
+            !vla::make_tmap_bf16(&ld.tm_o224, ld.w_o, D, p->qc, p->qc, 224) ||
+            !vla::make_tmap_bf16(&ld.tm_d224, ld.w_d, D, p->F_pad, p->F_pad, 224) ||
             !vla::make_tmap_bf16(&ld.tm_gu, ld.w_gu, 2 * p->F_pad, D, D, kBN) ||
             !vla::make_tmap_bf16(&ld.tm_d, ld.w_d, D, p->F_pad, p->F_pad, kBN)) {
             free_prefix(p);
@@ -504,11 +507,15 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
     // QKV tile width: the one with fewer column-slots in its last wave of tiles (waves x width;
     // 192 pays where 256-wide tiles leave a mostly idle second wave, e.g. 1024 tokens of a 7B
     // block: 192 tiles of 256 on 152 SMs, 256 tiles of 192), 256 on a tie
-    auto wave_cost = [&](int bn) {
-        const long long tiles = (long long)((M + 127) / 128) * ((p->qkv_n + bn - 1) / bn);
+    // The same choice for the O and down projections (N = D) between 256 and 224 columns
+    // (1024 tokens: 128 tiles of 256 leave 24 SMs idle, 152 tiles of 224 fill them).
+    auto wave_cost = [&](int n, int bn) {
+        const long long tiles = (long long)((M + 127) / 128) * ((n + bn - 1) / bn);
         return ((tiles + p->num_sms - 1) / p->num_sms) * bn;
     };
-    const int qkv_bn = wave_cost(192) < wave_cost(kBN) ? 192 : kBN;
+    const int qkv_bn = wave_cost(p->qkv_n, 192) < wave_cost(p->qkv_n, kBN) ? 192 : kBN;
+    const int d_bn = wave_cost(D, 224) < wave_cost(D, kBN) ? 224 : kBN;
+    const int ss_w = d_bn == kBN ? 256 : 32;  // row-statistics partials: one per tile or per 32 columns
     for (int l = layer_begin; l < layer_end && e == cudaSuccess; ++l) {
         const LayerDev& ld = p->layers[l];
         const bf16* x = (l == layer_begin) ? (const bf16*)hidden_in : (const bf16*)hidden_out;
@@ -517,7 +524,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         // block's down-projection epilogue) + QKV projection + RoPE + KV write
         if (l == layer_begin) {
             stage_mark(p, VLA_STAGE_ROWSTAT, true);
-            e = vla::launch_row_sumsq(x, M, D, D, p->ws_ss_x, stream, pdl(VLA_STAGE_ROWSTAT));
+            e = vla::launch_row_sumsq(x, M, D, D, ss_w, p->ws_ss_x, stream, pdl(VLA_STAGE_ROWSTAT));
             stage_mark(p, VLA_STAGE_ROWSTAT, false);
             if (e != cudaSuccess) break;
             ++launches;
@@ -528,7 +535,8 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ep.out = p->ws_q;
         ep.ld_out = p->qc;
         ep.ss_in = p->ws_ss_x;
-        ep.ss_chunks = D / 256;
+        ep.ss_width = ss_w;
+        ep.ss_groups = D / ss_w;
         ep.norm_dim = D;
         ep.eps = eps;
         ep.kcache = kv->k_plane(l);
@@ -575,11 +583,12 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         eo.resid = x;
         eo.ld_resid = D;
         eo.ss_out = p->ws_ss_mid;
-        eo.ss_chunks = D / 256;
+        eo.ss_width = ss_w;
+        eo.ss_groups = D / ss_w;
         eo.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_O, true);
-        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_attn, ld.tm_o, M, D, p->qc, eo, p->num_sms, stream,
-                             pdl(VLA_STAGE_GEMM_O));
+        e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_attn, d_bn == 224 ? ld.tm_o224 : ld.tm_o, M, D, p->qc, eo,
+                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_O));
         stage_mark(p, VLA_STAGE_GEMM_O, false);
         if (e != cudaSuccess) break;
         // RMSNorm (row statistics from the O epilogue) + gate/up + SwiGLU
@@ -589,7 +598,8 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         eg.out = p->ws_m;
         eg.ld_out = p->F_pad;
         eg.ss_in = p->ws_ss_mid;
-        eg.ss_chunks = D / 256;
+        eg.ss_width = ss_w;
+        eg.ss_groups = D / ss_w;
         eg.norm_dim = D;
         eg.eps = eps;
         eg.status = p->d_status;
@@ -608,11 +618,12 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ed.ld_resid = D;
         ed.ss_out = (l + 1 < layer_end) ? p->ws_ss_x : nullptr;  // the next block's row statistics
         ed.out_host = (l + 1 == layer_end) ? host_dev : nullptr;   // h^(layer_end) straight to the host
-        ed.ss_chunks = D / 256;
+        ed.ss_width = ss_w;
+        ed.ss_groups = D / ss_w;
         ed.status = p->d_status;
         stage_mark(p, VLA_STAGE_GEMM_DOWN, true);
-        e = vla::launch_gemm(vla::kEpiResid, kBN, tm_m, ld.tm_d, M, D, p->F_pad, ed, p->num_sms, stream,
-                             pdl(VLA_STAGE_GEMM_DOWN));
+        e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_m, d_bn == 224 ? ld.tm_d224 : ld.tm_d, M, D, p->F_pad, ed,
+                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_DOWN));
         stage_mark(p, VLA_STAGE_GEMM_DOWN, false);
         launches += 5;
     }
