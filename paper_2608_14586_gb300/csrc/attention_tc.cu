@@ -2,25 +2,29 @@
 //
 // o[i, h] = sum_{j <= pos0 + i} softmax_j(q_ih . k_gj / sqrt(d_h)) v_gj,  g = h / (H / H_kv)
 //
-// Persistent: one CTA per SM (192 threads, 225 KB smem, all 512 TMEM columns) walks a list of
-// tiles (128 query rows of one head), numbered longest causal tile first and dealt to the CTAs
-// in a snake so that every CTA gets a similar number of key blocks.
-//   warp 0      TMA: each tile's Q into one of two Q buffers, then its K and V blocks of 128
-//               keys into two 2-stage rings (a K stage is released as soon as S has consumed
-//               it, a V stage after PV); one thread polls both rings and issues whichever load
-//               is free. K/V come from the layer's cache through a 3-D tensor map whose key
-//               extent ends at the context length, so keys past it arrive as zeros.
-//   warp 1      TMEM allocation; one thread issues S = Q K^T (M=128, N=128 keys, K=d_h) into
-//               one of two TMEM S buffers, and O += P V (M=128, N=d_h, K=128 keys) with P from
-//               shared memory (K-major) and V as an MN-major operand, into one of two TMEM O
-//               accumulators (alternating by tile, so a tile's epilogue overlaps the next).
-//   warps 2..5  softmax, one thread per query row (TMEM lane): reads its S row once with
-//               tcgen05.ld, masks, takes the row max, writes P = exp2(s - m) as bf16 into a
-//               128-byte-swizzled shared tile, keeps the row sum; rescales its O row in TMEM
-//               only when the running max grows by more than 2^8 (otherwise the stale max is
-//               exact arithmetic with values up to 2^8); then the tile's O / l to global memory.
-// The ring and buffer phases run on per-CTA block and tile counters across tiles. Every wait
-// is bounded.
+// Persistent: one CTA per SM (320 threads, all 512 TMEM columns) walks a list of work units,
+// each a PAIR of query tiles of one head (tile A = 128 query rows, tile B = the next 128),
+// numbered longest first and dealt to the CTAs in a snake so every CTA gets a similar number
+// of key blocks. Both tiles read the same key/value blocks, which are loaded once for the pair.
+//   warp 0      TMA: the pair's two Q tiles, then K and V blocks of 128 keys through two 2-stage
+//               rings shared by the two tiles. K/V come from the layer's cache through a 3-D
+//               tensor map whose key extent ends at the context length, so keys past it arrive
+//               as zeros.
+//   warp 1      TMEM allocation; one thread issues, per tile t, S_t = Q_t K^T (M=128, N=128
+//               keys, K=d_h) into TMEM columns [128t, 128t+128) and O_t += P_t V (M=128, N=d_h,
+//               K=128 keys) into TMEM columns [256 + t*d_h, ...), with P_t read from tensor
+//               memory (the softmax writes it as packed bf16 over the first 64 columns of S_t)
+//               and V from shared memory as an MN-major operand. The next S_t is issued once
+//               PV_t has completed, since P_t occupies its columns.
+//   warps 2..5  softmax of tile A, warps 6..9 of tile B; one thread per query row (TMEM lane):
+//               reads its S row once (tcgen05.ld), masks, takes the row max, writes
+//               P = exp2(s - m) as bf16 into tensor memory (tcgen05.st), keeps the row sum, and
+//               rescales its O row only when the running max grows by more than 2^8 (a stale max
+//               below that is exact arithmetic with values up to 2^8). Each tile is a chain
+//               S -> softmax -> PV -> next S; the two chains of a pair run side by side, so
+//               the tensor core works on one tile while the other's softmax runs. At the end of
+//               a pair each group writes its tile's O / l.
+// Phases of every barrier follow per-CTA block and pair counters. Every wait is bounded.
 #include "common.cuh"
 #include "internal.h"
 
@@ -30,35 +34,31 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;
 
 template <int DH>
 struct AttnCfg {
-    static constexpr int KCH = DH / 64;                 // 64-wide head-dim chunks
-    static constexpr uint32_t CHUNK = 128 * 64 * 2;     // one [128 rows][64] bf16 chunk
+    static constexpr int KCH = DH / 64;              // 64-wide head-dim chunks
+    static constexpr uint32_t CHUNK = 128 * 64 * 2;  // one [128 rows][64] bf16 chunk
     static constexpr uint32_t Q_BYTES = KCH * CHUNK;
     static constexpr uint32_t KV_BYTES = KCH * CHUNK;
-    static constexpr uint32_t P_BYTES = 2 * CHUNK;       // 128 keys = 2 chunks of 64
     static constexpr int K_STAGES = 2;
     static constexpr int V_STAGES = 2;
-    // Q is double-buffered across the CTA's tiles; one P tile suffices because PV(j) is
-    // issued as soon as P(j) is written
-    static constexpr uint32_t OFF_K = 2 * Q_BYTES;
+    static constexpr uint32_t OFF_K = 2 * Q_BYTES;  // Q of tile A, then of tile B
     static constexpr uint32_t OFF_V = OFF_K + K_STAGES * KV_BYTES;
-    static constexpr uint32_t OFF_P = OFF_V + V_STAGES * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_V + V_STAGES * KV_BYTES;
     static constexpr uint32_t SMEM = OFF_BAR + 256 + 1024;
-    // S0 [0,128) S1 [128,256), then two O accumulators of DH columns (one per tile in flight)
     static constexpr uint32_t TMEM_COLS = 512;
-    static constexpr uint32_t O_COL = 256;
+    static constexpr uint32_t O_COL = 256;  // O of tile t at O_COL + t * DH
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(kBM, kBN);
     static constexpr uint32_t IDESC_O = idesc_bf16_f32_bmn(kBM, DH);
 };
 
 struct Bars {
-    uint64_t q_full[2], q_free[2], k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2], p_full,
-        p_free, o_full[2], o_free[2], mma_done;
+    uint64_t q_full, q_free, k_full[2], k_empty[2], v_full[2], v_empty[2];
+    uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];  // per tile
+    uint64_t mma_done;
     uint32_t tmem_slot;
 };
 
@@ -79,25 +79,27 @@ struct TcAttnArgs {
     unsigned* status;
 };
 
-// One causal tile: 128 query rows of one head, and the key blocks it needs.
-struct Tile {
-    int mt, h, g, m0, nblk;
+// A pair of query tiles of one head: tile A at rows [m0, m0+128), tile B at [m0+128, m0+256)
+// (absent when m0 + 128 >= M), and the key blocks each needs.
+struct Pair {
+    int h, g, m0, n[2];  // n[1] == 0: no tile B
 };
 
-// The CTA's k-th tile, or false. Tiles are numbered longest first (every head of the latest
-// query tile, then the next query tile, ...) and dealt to the persistent CTAs in a snake
-// (round r: CTA c takes tile r*G + c on even rounds, (r+1)*G - 1 - c on odd ones), so each CTA
-// gets a mix of long and short causal tiles.
-VLA_DEV bool cta_tile(int k, int num_m, const TcAttnArgs& a, Tile& t) {
+// The CTA's k-th pair, or false. Pairs are numbered longest first (every head of the latest
+// pair of query tiles, then the next, ...) and dealt to the persistent CTAs in a snake
+// (round r: CTA c takes unit r*G + c on even rounds, (r+1)*G - 1 - c on odd ones).
+VLA_DEV bool cta_pair(int k, int num_p, const TcAttnArgs& a, Pair& p) {
     const int G = gridDim.x, c = blockIdx.x;
     const int idx = (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
-    if (idx >= num_m * a.H) return false;
-    t.mt = num_m - 1 - idx / a.H;
-    t.h = idx % a.H;
-    t.g = t.h / (a.H / a.Hkv);
-    t.m0 = t.mt * kBM;
-    const int key_end = a.pos0 + min(t.m0 + kBM, a.M);
-    t.nblk = (key_end + kBN - 1) / kBN;
+    if (idx >= num_p * a.H) return false;
+    const int pm = num_p - 1 - idx / a.H;
+    p.h = idx % a.H;
+    p.g = p.h / (a.H / a.Hkv);
+    p.m0 = pm * 2 * kBM;
+    for (int t = 0; t < 2; ++t) {
+        const int r0 = p.m0 + t * kBM;
+        p.n[t] = r0 < a.M ? (a.pos0 + min(r0 + kBM, a.M) + kBN - 1) / kBN : 0;
+    }
     return true;
 }
 
@@ -113,23 +115,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_m = (a.M + kBM - 1) / kBM;
+    const int num_p = (a.M + 2 * kBM - 1) / (2 * kBM);
 
     if (threadIdx.x == 0) {
+        mbar_init(&bars->q_full, 1);
+        mbar_init(&bars->q_free, 1);
         for (int b = 0; b < 2; ++b) {
-            mbar_init(&bars->q_full[b], 1);
-            mbar_init(&bars->q_free[b], 1);
-            mbar_init(&bars->k_full[b], 1);
-            mbar_init(&bars->k_empty[b], 1);
             mbar_init(&bars->v_full[b], 1);
             mbar_init(&bars->v_empty[b], 1);
+            mbar_init(&bars->k_full[b], 1);
+            mbar_init(&bars->k_empty[b], 1);
             mbar_init(&bars->s_full[b], 1);
-            mbar_init(&bars->s_free[b], 128);
-            mbar_init(&bars->o_full[b], 1);
+            mbar_init(&bars->p_full[b], 128);
+            mbar_init(&bars->pv_done[b], 1);
             mbar_init(&bars->o_free[b], 128);
         }
-        mbar_init(&bars->p_full, 128);
-        mbar_init(&bars->p_free, 1);
         mbar_init(&bars->mma_done, 1);
         s_abort = 0;
         fence_barrier_init();
@@ -153,37 +153,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer ----------------
-            // ring slot of global block n: n % 2, phase (n / 2) & 1 (K and V alike; Q by tile)
+            // ring slot of global block n: n % 2, phase (n / 2) & 1 (K and V alike)
             bool ok = true;
-            uint32_t issued_k = 0, issued_v = 0, issued_q = 0, ph_k = 0, ph_v = 0, ph_q = 0;
-            uint32_t nk = 0, nv = 0;  // K / V blocks issued so far (all tiles)
-            Tile t;
+            uint32_t issued_k = 0, issued_v = 0, ph_k = 0, ph_v = 0;
+            bool issued_q = false;
+            uint32_t ph_q = 0;
+            uint32_t nk = 0, nv = 0;  // K / V blocks issued so far (all pairs)
+            Pair p;
             long long t0 = clock64();
-            for (int k = 0; ok && cta_tile(k, num_m, a, t); ++k) {
-                const int qb = k & 1;
-                const uint32_t qn = (uint32_t)(k >> 1);
-                if (!wait_ab(&bars->q_free[qb], (qn & 1u) ^ 1u, &s_abort)) {
+            for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
+                if (!wait_ab(&bars->q_free, ((uint32_t)k & 1u) ^ 1u, &s_abort)) {
                     ok = false;
                     break;
                 }
-                mbar_arrive_expect_tx(&bars->q_full[qb], C::Q_BYTES);
-                for (int c = 0; c < C::KCH; ++c)
-                    tma_load_2d(smem + qb * C::Q_BYTES + c * C::CHUNK, &tmQ, &bars->q_full[qb], t.h * DH + c * 64,
-                                t.m0);
-                issued_q |= 1u << qb;
-                ph_q = (ph_q & ~(1u << qb)) | ((qn & 1u) << qb);
+                const int ntiles = p.n[1] > 0 ? 2 : 1;
+                mbar_arrive_expect_tx(&bars->q_full, C::Q_BYTES * ntiles);
+                for (int t = 0; t < ntiles; ++t)
+                    for (int c = 0; c < C::KCH; ++c)
+                        tma_load_2d(smem + t * C::Q_BYTES + c * C::CHUNK, &tmQ, &bars->q_full, p.h * DH + c * 64,
+                                    p.m0 + t * kBM);
+                issued_q = true;
+                ph_q = (uint32_t)k & 1u;
+                const int nmax = max(p.n[0], p.n[1]);
                 int jk = 0, jv = 0;
                 t0 = clock64();
-                while (jk < t.nblk || jv < t.nblk) {
+                while (jk < nmax || jv < nmax) {
                     bool progressed = false;
-                    if (jk < t.nblk) {
+                    if (jk < nmax) {
                         const int b = nk & 1;
                         const uint32_t n = nk >> 1;
                         if (mbar_try_wait(&bars->k_empty[b], (n & 1u) ^ 1u)) {
                             mbar_arrive_expect_tx(&bars->k_full[b], C::KV_BYTES);
                             for (int c = 0; c < C::KCH; ++c)
                                 tma_load_3d(smem + C::OFF_K + b * C::KV_BYTES + c * C::CHUNK, &tmK, &bars->k_full[b],
-                                            c * 64, jk * kBN, t.g);
+                                            c * 64, jk * kBN, p.g);
                             issued_k |= 1u << b;
                             ph_k = (ph_k & ~(1u << b)) | ((n & 1u) << b);
                             ++jk;
@@ -191,14 +194,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                             progressed = true;
                         }
                     }
-                    if (jv < t.nblk && jv < jk) {
+                    if (jv < nmax) {  // V runs ahead of K as far as its ring allows
                         const int b = nv & 1;
                         const uint32_t n = nv >> 1;
                         if (mbar_try_wait(&bars->v_empty[b], (n & 1u) ^ 1u)) {
                             mbar_arrive_expect_tx(&bars->v_full[b], C::KV_BYTES);
                             for (int c = 0; c < C::KCH; ++c)
                                 tma_load_3d(smem + C::OFF_V + b * C::KV_BYTES + c * C::CHUNK, &tmV, &bars->v_full[b],
-                                            c * 64, jv * kBN, t.g);
+                                            c * 64, jv * kBN, p.g);
                             issued_v |= 1u << b;
                             ph_v = (ph_v & ~(1u << b)) | ((n & 1u) << b);
                             ++jv;
@@ -219,8 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 set_status(a.status, kDevTimeout);
             }
             // every copy this thread issued lands before the CTA can exit
+            if (issued_q) mbar_wait(&bars->q_full, ph_q);
             for (int b = 0; b < 2; ++b) {
-                if (issued_q & (1u << b)) mbar_wait(&bars->q_full[b], (ph_q >> b) & 1u);
                 if (issued_k & (1u << b)) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
                 if (issued_v & (1u << b)) mbar_wait(&bars->v_full[b], (ph_v >> b) & 1u);
             }
@@ -229,60 +232,85 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
             bool ok = true;
-            uint32_t gb = 0;  // global block counter (S buffers, K/V rings, P)
-            // PV of global block n for a tile whose O accumulator is ob (first: no accumulate)
-            auto issue_pv = [&](uint32_t n, int ob, bool first) -> bool {
-                const int vb = n & 1;
-                if (!wait_ab(&bars->p_full, n & 1u, &s_abort)) return false;
-                if (!wait_ab(&bars->v_full[vb], (n >> 1) & 1u, &s_abort)) return false;
-                tc_fence_after();
-                const uint32_t sP = smem_u32(smem + C::OFF_P);
-                const uint32_t sV = smem_u32(smem + C::OFF_V + vb * C::KV_BYTES);
+            uint32_t gt[2] = {0, 0};  // blocks of tile slot t so far (S, P, PV phases)
+            uint32_t et[2] = {0, 0};  // pairs in which tile slot t existed (O phases)
+            uint32_t nkv = 0;         // K/V blocks so far (ring phases)
+            auto issue_s = [&](int t, uint32_t n, uint32_t sQ) {
+                const uint32_t sK = smem_u32(smem + C::OFF_K + (n & 1) * C::KV_BYTES);
 #pragma unroll
-                for (int kk = 0; kk < kBN / 16; ++kk) {
-                    const uint64_t ad = sw128_kmajor_desc(sP + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                    const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
-                    umma_bf16_ss(tmem + C::O_COL + ob * DH, ad, bd, C::IDESC_O, (!first || kk > 0) ? 1u : 0u);
+                for (int kk = 0; kk < DH / 16; ++kk) {
+                    const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
+                    const uint64_t bd = sw128_kmajor_desc(sK + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
+                    umma_bf16_ss(tmem + t * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(&bars->p_free);
-                umma_commit(&bars->v_empty[vb]);
-                return true;
+                umma_commit(&bars->s_full[t]);
             };
-            Tile t;
-            for (int k = 0; ok && cta_tile(k, num_m, a, t); ++k) {
-                const int qb = k & 1, ob = k & 1;
-                const uint32_t qn = (uint32_t)(k >> 1);
-                // Q of this tile landed, and the O accumulator's previous tile (k-2) was read out
-                if (!wait_ab(&bars->q_full[qb], qn & 1u, &s_abort) ||
-                    !wait_ab(&bars->o_free[ob], (qn & 1u) ^ 1u, &s_abort)) {
+            Pair p;
+            for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
+                const int nmax = max(p.n[0], p.n[1]);
+                if (!wait_ab(&bars->q_full, (uint32_t)k & 1u, &s_abort) ||
+                    !wait_ab(&bars->k_full[nkv & 1], (nkv >> 1) & 1u, &s_abort)) {
                     ok = false;
                     break;
                 }
-                const uint32_t sQ = smem_u32(smem + qb * C::Q_BYTES);
-                for (int j = 0; j < t.nblk && ok; ++j) {
-                    const uint32_t n = gb + j;
-                    const int b = n & 1;
-                    if (!wait_ab(&bars->k_full[b], (n >> 1) & 1u, &s_abort) ||
-                        !wait_ab(&bars->s_free[b], ((n >> 1) & 1u) ^ 1u, &s_abort)) {
+                tc_fence_after();
+                // S of block 0 for both tiles (their S columns were freed by the previous pair's
+                // last PV, which this thread waited for before issuing anything after it)
+                for (int t = 0; t < 2; ++t)
+                    if (p.n[t] > 0) issue_s(t, nkv, smem_u32(smem + t * C::Q_BYTES));
+                umma_commit(&bars->k_empty[nkv & 1]);
+                if (nmax == 1) umma_commit(&bars->q_free);
+                for (int j = 0; j < nmax && ok; ++j) {
+                    const uint32_t n = nkv + j;
+                    if (!wait_ab(&bars->v_full[n & 1], (n >> 1) & 1u, &s_abort)) {
                         ok = false;
                         break;
                     }
-                    tc_fence_after();
-                    const uint32_t sK = smem_u32(smem + C::OFF_K + b * C::KV_BYTES);
+                    bool k_next = false;  // K of block j+1 waited for
+                    for (int t = 0; t < 2 && ok; ++t) {
+                        if (j >= p.n[t]) continue;
+                        if (!wait_ab(&bars->p_full[t], gt[t] & 1u, &s_abort) ||
+                            (j == 0 && !wait_ab(&bars->o_free[t], (et[t] & 1u) ^ 1u, &s_abort))) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t sV = smem_u32(smem + C::OFF_V + (n & 1) * C::KV_BYTES);
 #pragma unroll
-                    for (int kk = 0; kk < DH / 16; ++kk) {
-                        const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                        const uint64_t bd = sw128_kmajor_desc(sK + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                        umma_bf16_ss(tmem + b * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
+                        for (int kk = 0; kk < kBN / 16; ++kk) {
+                            const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
+                            umma_bf16_ts(tmem + C::O_COL + t * DH, tmem + t * kBN + kk * 8, bd, C::IDESC_O,
+                                         (j > 0 || kk > 0) ? 1u : 0u);
+                        }
+                        umma_commit(&bars->pv_done[t]);
+                        if (j + 1 < p.n[t]) {
+                            // the next S of this tile overwrites P: wait for this PV, and for K
+                            if (!wait_ab(&bars->pv_done[t], gt[t] & 1u, &s_abort) ||
+                                (!k_next && !wait_ab(&bars->k_full[(n + 1) & 1], ((n + 1) >> 1) & 1u, &s_abort))) {
+                                ok = false;
+                                break;
+                            }
+                            k_next = true;
+                            tc_fence_after();
+                            issue_s(t, n + 1, smem_u32(smem + t * C::Q_BYTES));
+                        }
+                        ++gt[t];
                     }
-                    umma_commit(&bars->s_full[b]);
-                    umma_commit(&bars->k_empty[b]);
-                    if (j == t.nblk - 1) umma_commit(&bars->q_free[qb]);  // the tile's last read of Q
-                    if (j >= 1 && !issue_pv(n - 1, ob, j == 1)) ok = false;
+                    if (!ok) break;
+                    umma_commit(&bars->v_empty[n & 1]);
+                    if (j + 1 < nmax) {
+                        umma_commit(&bars->k_empty[(n + 1) & 1]);
+                        if (j + 2 == nmax) umma_commit(&bars->q_free);  // the pair's last S was just issued
+                    }
                 }
-                if (ok && !issue_pv(gb + t.nblk - 1, ob, t.nblk == 1)) ok = false;
-                if (ok) umma_commit(&bars->o_full[ob]);
-                gb += t.nblk;
+                if (!ok) break;
+                // the last PV of each tile must finish before that tile's S columns are reused
+                for (int t = 0; t < 2 && ok; ++t) {
+                    if (p.n[t] == 0) continue;
+                    if (!wait_ab(&bars->pv_done[t], (gt[t] - 1) & 1u, &s_abort)) ok = false;
+                    ++et[t];
+                }
+                nkv += nmax;
             }
             if (!ok) {
                 s_abort = 1;
@@ -293,114 +321,100 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait(&bars->mma_done, 0);
         }
     } else {
-        // ---------------- softmax / correction / epilogue (warps 2..5) ----------------
+        // ---------------- softmax / correction / epilogue: tile A (warps 2..5), B (6..9) ----------------
+        const int t = (warp - 2) >> 2;
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t scol = (uint32_t)t * kBN;
+        const uint32_t ocol = C::O_COL + (uint32_t)t * DH;
         bool ok = true;
-        uint32_t gb = 0;
-        Tile t;
-        for (int k = 0; ok && cta_tile(k, num_m, a, t); ++k) {
-            const int ob = k & 1;
-            const uint32_t ocol = C::O_COL + ob * DH;
-            const int qpos = a.pos0 + t.m0 + row;
-            const int min_qpos = a.pos0 + t.m0;
+        uint32_t g = 0;  // blocks of this tile slot so far
+        Pair p;
+        for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
+            if (p.n[t] == 0) continue;  // no tile B in this pair
+            const int m0 = p.m0 + t * kBM;
+            const int qpos = a.pos0 + m0 + row;
+            const int min_qpos = a.pos0 + m0;
             float m_run = -INFINITY, l_run = 0.f;
-            for (int j = 0; j < t.nblk; ++j) {
-                const uint32_t n = gb + j;
-                const int b = n & 1;
-                const int kb = j * kBN;
-                const bool need_mask = (kb + kBN - 1 > min_qpos) || (kb + kBN > a.ctx);
-                ok = wait_ab(&bars->s_full[b], (n >> 1) & 1u, &s_abort);
-                __syncwarp();
-                if (!__all_sync(0xFFFFFFFFu, ok)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                // the whole S row (128 keys) in registers; row max of the raw masked scores
+            for (int j = 0; j < p.n[t]; ++j) {
                 uint32_t sr[kBN];
-                tmem_ld128(trow + b * kBN, sr);
-                if (need_mask) {
-#pragma unroll
-                    for (int i = 0; i < kBN; ++i) {
-                        const int key = kb + i;
-                        if (key > qpos || key >= a.ctx) sr[i] = 0xFF800000u;  // -inf
-                    }
-                }
-                // row max in 8 independent chains, then combined
-                float mc[8];
-#pragma unroll
-                for (int q = 0; q < 8; ++q) mc[q] = __uint_as_float(sr[q]);
-#pragma unroll
-                for (int i = 8; i < kBN; ++i) mc[i & 7] = fmaxf(mc[i & 7], __uint_as_float(sr[i]));
-                const float mraw = fmaxf(fmaxf(fmaxf(mc[0], mc[1]), fmaxf(mc[2], mc[3])),
-                                         fmaxf(fmaxf(mc[4], mc[5]), fmaxf(mc[6], mc[7])));
-                const float mx = mraw * a.scale_log2;  // scale > 0
                 float m_new = m_run;
                 bool need = false;
-                if (m_run == -INFINITY) {
-                    m_new = mx;
-                } else if (mx > m_run + kRescaleLog2) {
-                    need = true;
-                    m_new = mx;
-                }
-                const float corr = need ? ex2_approx(m_run - m_new) : 1.f;
-                l_run *= corr;
-                const bool warp_need = __any_sync(0xFFFFFFFFu, need);
-                // the P tile was last read by PV of the previous global block
-                if (n >= 1) ok = wait_ab(&bars->p_free, (n - 1) & 1u, &s_abort);
-                if (!__all_sync(0xFFFFFFFFu, ok)) {
-                    ok = false;
-                    break;
-                }
-                // P = exp2(s * scale - m) -> bf16 in the 128-byte-swizzled K-major tile
-                uint8_t* prow = smem + C::OFF_P + row * 128;
-                const float neg_m = -m_new;
-                float ls[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums of the row
-#pragma unroll
-                for (int c = 0; c < kBN / 8; ++c) {  // 16-byte chunks of 8 keys
-                    uint32_t pk[4];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float p0 = ex2_approx(fmaf(__uint_as_float(sr[8 * c + 2 * q]), a.scale_log2, neg_m));
-                        const float p1 = ex2_approx(fmaf(__uint_as_float(sr[8 * c + 2 * q + 1]), a.scale_log2, neg_m));
-                        ls[q] += p0 + p1;
-                        pk[q] = pack_bf16x2(p0, p1);
-                    }
-                    // keys [8c, 8c+8): 64-key half c/8, 16-byte chunk c%8, swizzled by the row
-                    uint8_t* half = prow + (c >> 3) * C::CHUNK;
-                    *reinterpret_cast<uint4*>(half + (((c & 7) ^ (row & 7)) << 4)) =
-                        make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                }
-                l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-                tc_fence_before();
-                mbar_arrive(&bars->s_free[b]);
-                if (warp_need) {
-                    // O must hold PV of the previous block before it is rescaled (j >= 1 here)
-                    ok = wait_ab(&bars->p_free, (n - 1) & 1u, &s_abort);
+                {
+                    const int kb = j * kBN;
+                    const bool need_mask = (kb + kBN - 1 > min_qpos) || (kb + kBN > a.ctx);
+                    ok = wait_ab(&bars->s_full[t], g & 1u, &s_abort);
+                    __syncwarp();
                     if (!__all_sync(0xFFFFFFFFu, ok)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-#pragma unroll 1
-                    for (int c = 0; c < DH / 32; ++c) {
-                        uint32_t r[32];
-                        tmem_ld32(trow + ocol + c * 32, r);
+                    tmem_ld128(trow + scol, sr);
+                    if (need_mask) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * corr);
-                        tmem_st32(trow + ocol + c * 32, r);
+                        for (int i = 0; i < kBN; ++i) {
+                            const int key = kb + i;
+                            if (key > qpos || key >= a.ctx) sr[i] = 0xFF800000u;  // -inf
+                        }
+                    }
+                    float mc[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) mc[q] = __uint_as_float(sr[q]);
+#pragma unroll
+                    for (int i = 8; i < kBN; ++i) mc[i & 7] = fmaxf(mc[i & 7], __uint_as_float(sr[i]));
+                    const float mraw = fmaxf(fmaxf(fmaxf(mc[0], mc[1]), fmaxf(mc[2], mc[3])),
+                                             fmaxf(fmaxf(mc[4], mc[5]), fmaxf(mc[6], mc[7])));
+                    const float mx = mraw * a.scale_log2;  // scale > 0
+                    if (m_run == -INFINITY) {
+                        m_new = mx;
+                    } else if (mx > m_run + kRescaleLog2) {
+                        need = true;
+                        m_new = mx;
                     }
                 }
-                fence_proxy_async_smem();
-                tc_fence_before();
-                mbar_arrive(&bars->p_full);
-                m_run = m_new;
+                {
+                    const float corr = need ? ex2_approx(m_run - m_new) : 1.f;
+                    l_run *= corr;
+                    const bool warp_need = __any_sync(0xFFFFFFFFu, need);
+                    // P = exp2(s * scale - m) as packed bf16 over the first 64 columns of S
+                    const float neg_m = -m_new;
+                    float ls[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums of the row
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t pk[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const float p0 = ex2_approx(fmaf(__uint_as_float(sr[64 * h + 2 * i]), a.scale_log2, neg_m));
+                            const float p1 =
+                                ex2_approx(fmaf(__uint_as_float(sr[64 * h + 2 * i + 1]), a.scale_log2, neg_m));
+                            ls[i & 3] += p0 + p1;
+                            pk[i] = pack_bf16x2(p0, p1);
+                        }
+                        tmem_st32(trow + scol + 32 * h, pk);
+                    }
+                    l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+                    if (warp_need) {
+                        // PV of the previous block has completed: this block's S was issued after it
+#pragma unroll 1
+                        for (int c = 0; c < DH / 32; ++c) {
+                            uint32_t r[32];
+                            tmem_ld32(trow + ocol + c * 32, r);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * corr);
+                            tmem_st32(trow + ocol + c * 32, r);
+                        }
+                    }
+                    tc_fence_before();
+                    mbar_arrive(&bars->p_full[t]);
+                    m_run = m_new;
+                    ++g;
+                }
             }
             if (!ok) break;
-            // epilogue of this tile (overlaps the first S blocks of the next one)
-            ok = wait_ab(&bars->o_full[ob], (uint32_t)(k >> 1) & 1u, &s_abort);
+            // epilogue of this tile: after its last PV
+            ok = wait_ab(&bars->pv_done[t], (g - 1) & 1u, &s_abort);
             __syncwarp();
             if (!__all_sync(0xFFFFFFFFu, ok)) {
                 ok = false;
@@ -408,8 +422,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-            const bool row_ok = (t.m0 + row) < a.M;
-            bf16* orow = a.out + (size_t)(t.m0 + row) * a.ld_out + t.h * DH;
+            const bool row_ok = (m0 + row) < a.M;
+            bf16* orow = a.out + (size_t)(m0 + row) * a.ld_out + p.h * DH;
 #pragma unroll 1
             for (int c = 0; c < DH / 32; ++c) {
                 uint32_t r[32];
@@ -425,8 +439,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             tc_fence_before();
-            mbar_arrive(&bars->o_free[ob]);
-            gb += t.nblk;
+            mbar_arrive(&bars->o_free[t]);
         }
         if (!ok) {
             s_abort = 1;
@@ -468,7 +481,7 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
     a.scale_log2 = p.scale_log2;
     a.out = p.out;
     a.status = status;
-    // persistent: one CTA per SM (tensor-memory kernels get one per SM), each walking its tiles
+    // persistent: one CTA per SM (tensor-memory kernels get one per SM), each walking its pairs
     static int sms = 0;
     if (!sms) {
         int dev = 0;
@@ -476,8 +489,8 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (sms <= 0) sms = 1;
     }
-    const int tiles = ((p.M + kBM - 1) / kBM) * p.H;
-    const dim3 grid(tiles < sms ? tiles : sms);
+    const int units = ((p.M + 2 * kBM - 1) / (2 * kBM)) * p.H;
+    const dim3 grid(units < sms ? units : sms);
     return launch_ex(attn_prefill_tc_kernel<DH>, grid, dim3(kThreads), C::SMEM, stream, pdl, tq, tk, tv, a);
 }
 

@@ -89,12 +89,10 @@ cudaError_t launch_attn_prefill_tc(const AttnPrefillParams& p, unsigned* status,
 // ---------------------------------------------------------------------------------------
 // Elementwise / setup kernels
 // ---------------------------------------------------------------------------------------
-// ss[i][t] = sum over columns [256t, 256t+256) of x[i][c]^2 in fp32, formed as 8 in-order chains
-// over 32-column groups added in group order: the same partial sums the residual GEMM epilogue
-// writes for its output, so a block gets bit-identical row statistics whether its input came
-// from the previous block or from the caller.
-// ss[row][t] = the row's sum of squares over columns [t*width, (t+1)*width), in the order
-// EpiParams describes (width 256 or 32)
+// ss[row][t] = the row's sum of squares over columns [t*width, (t+1)*width) (width 256 or 32),
+// in the order EpiParams describes: the same partial sums the residual GEMM epilogue writes
+// for its output, so a block gets bit-identical row statistics whether its input came from
+// the previous block or from the caller.
 cudaError_t launch_row_sumsq(const bf16* x, int M, int D, int ld, int width, float* ss, cudaStream_t stream,
                              bool pdl = false);
 
