@@ -11,9 +11,10 @@
 //   3. One thread per key row reads its G scores, the CTA takes the per-head max and sum of
 //      exp2(s * log2(e)/sqrt(d_h) - max), and writes P^T (bf16, 128-byte-swizzled K-major).
 //   4. O^T = V^T P^T on tcgen05 (M = d_h, N = 16, K = keys; V^T read MN-major in place).
-//   5. The CTA's (max, sum, unnormalised O) go to shared memory; after a cluster barrier CTA r
-//      merges output elements [r*G*d_h/cs, (r+1)*G*d_h/cs) over the cluster through
-//      distributed shared memory in fixed rank order and writes them as bf16.
+//   5. Each CTA stores its (max, sum, unnormalised O) through distributed shared memory into
+//      the inbox of the rank that merges each element slice; after one cluster barrier CTA r
+//      merges output elements [r*G*d_h/cs, (r+1)*G*d_h/cs) from its inbox in fixed rank order
+//      and writes them as bf16.
 // Every mbarrier wait is bounded; a timeout sets the status word and the kernel winds down.
 #include "common.cuh"
 #include "internal.h"
@@ -72,6 +73,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ float red_m[4][G], red_l[4][G];
     __shared__ float c_m[G], c_l[G];
     __shared__ __align__(16) float c_o[G * kDH];
+    // merge inbox: from each rank of the cluster, its (max, sum) per head and its unnormalised
+    // output over this CTA's element slice
+    __shared__ float rx_m[kMaxCs][G], rx_l[kMaxCs][G];
+    __shared__ float rx_o[kMaxCs][G * kDH / 8];
     __shared__ int s_ok;
     const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
     uint8_t* smem = smem_raw + pad;
@@ -278,8 +283,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_dealloc(tmem, kTmemCols);
     }
     if (!s_ok && tid == 0) set_status(p.status, kDevTimeout);
-    cluster_sync_all();  // every CTA's (c_m, c_l, c_o) is complete and visible to the cluster
+    // push this CTA's partial state to the rank that merges each element slice, then one
+    // cluster barrier (release / acquire) makes every inbox complete; nothing reads another
+    // CTA's shared memory after it, so no second barrier is needed before exit
     const int per_cta = G * kDH / p.cs;
+    for (int i = tid; i < p.cs * per_cta; i += kThreads) {
+        const int q = i / per_cta, k = i % per_cta;
+        st_dsmem_f32(&rx_o[rank][k], (uint32_t)q, c_o[q * per_cta + k]);
+    }
+    for (int i = tid; i < p.cs * G; i += kThreads) {
+        const int q = i / G, hh = i % G;
+        st_dsmem_f32(&rx_m[rank][hh], (uint32_t)q, c_m[hh]);
+        st_dsmem_f32(&rx_l[rank][hh], (uint32_t)q, c_l[hh]);
+    }
+    cluster_sync_all();
     if (tid < per_cta) {
         const int e = rank * per_cta + tid;
         const int hh = e / kDH;
@@ -287,9 +304,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int r = 0; r < kMaxCs; ++r) {
             if (r < p.cs) {
-                mr[r] = ld_dsmem_f32(&c_m[hh], (uint32_t)r);
-                lr[r] = ld_dsmem_f32(&c_l[hh], (uint32_t)r);
-                orr[r] = ld_dsmem_f32(&c_o[e], (uint32_t)r);
+                mr[r] = rx_m[r][hh];
+                lr[r] = rx_l[r][hh];
+                orr[r] = rx_o[r][tid];
             }
         }
         float mx = -INFINITY;
@@ -307,7 +324,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         p.out[((size_t)seq * p.H + kvh * G) * kDH + e] = __float2bfloat16_rn(ot / lt);
     }
-    cluster_sync_all();  // keep this CTA's shared memory alive until the cluster has read it
 }
 
 template <int G>

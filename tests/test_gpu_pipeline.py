@@ -79,6 +79,13 @@ def test_tiny_pipeline_per_frame_split_matches_oracle(vla_lib):
             got = oracle.bf16_to_f64(y)
             assert rel_l2(got, ref) < REL_L2_BLOCK
             assert cos_sim(got, ref) > COS_FINAL
+        # a pipeline destroyed with frames in flight finishes them first and frees everything
+        pl = vla.vla_pipeline_create(m.handle, cpu, M, 3)
+        for f in range(3):
+            vla.vla_pipeline_submit(pl, f, xs[f], M, splits[f], stream)
+        assert vla.vla_pipeline_in_flight(pl) == 3
+        vla.vla_pipeline_destroy(pl)
+        sync()
         assert vla.vla_last_async_error(m.handle) == 0
     finally:
         vla.vla_cpu_model_destroy(cpu)
@@ -108,6 +115,11 @@ def test_7b_pipeline_overlaps_gpu_prefix_with_cpu_suffix(vla_lib):
             with pytest.raises(vla.VlaError) as ei:
                 vla.vla_pipeline_submit(pl, 9, xs[2], M, 1, stream)  # below the CPU model's first block
             assert ei.value.name == "VLA_ERR_RANGE"
+            # frame 7's suffix (one CPU block over 512 tokens) is far from done right after submit
+            with pytest.raises(vla.VlaError) as ei:
+                vla.vla_pipeline_collect(pl, None, 0)
+            assert ei.value.name == "VLA_ERR_TIMEOUT"
+            assert vla.vla_pipeline_in_flight(pl) == 2  # a timed-out collect leaves the frame queued
             res = []
             for _ in range(2):
                 y = np.empty((M, s.hidden), dtype=np.uint16)
