@@ -468,18 +468,10 @@ cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMa
         }
     } else if (bn == 224) {
         if (ep.ss_out && ep.ss_width != 32) return cudaErrorInvalidValue;  // partials would straddle tiles
-        if (mode == kEpiResid || mode == kEpiPlain) return launch_one<224, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
+        if (mode == kEpiResid || mode == kEpiPlain)
+            return launch_one<224, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
     } else if (bn == 192) {
         if (mode == kEpiQKV) return launch_one<192, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
-    } else if (bn == 128) {
-        switch (mode) {
-            case kEpiPlain:
-            case kEpiResid:
-                if (ep.ss_out && ep.ss_width != 32) return cudaErrorInvalidValue;
-                return launch_one<128, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
-            case kEpiQKV: return cudaErrorInvalidValue;  // BN = 256 or 192 only
-            case kEpiSwiGLU: return cudaErrorInvalidValue;  // gate/up rows are interleaved for BN = 256
-        }
     }
     return cudaErrorInvalidValue;
 }

@@ -63,7 +63,8 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint6
 // for profilers and debuggers that serialise kernels anyway).
 bool pdl_enabled();
 
-// Launch: BN in {128, 256}. Returns a cudaError_t of the launch.
+// Launch with an N tile of bn columns: 256 (every mode), 224 (kEpiResid / kEpiPlain; row
+// statistics then per 32 columns) or 192 (kEpiQKV). Returns a cudaError_t of the launch.
 // pdl: programmatic dependent launch (the CTA prologue and the first weight-tile loads may
 // overlap the previous kernel; A and everything the epilogue reads come after the wait).
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
