@@ -9,9 +9,9 @@
 //     [panel][k][8] bf16, gains folded in and rounded to bf16 as on the GPU. The register
 //     tile is 12 rows x 8 columns: three 4-row vectors of A times each of the 8 weight values
 //     of a k step (24 fp32 vector accumulators; GCC vector extensions over 128-bit lanes: NEON
-//     on an Arm host, SSE on x86). A task tile is 96 rows x 128 columns over 256-deep k
+//     on an Arm host, SSE on x86). A task tile is 144 rows x 128 columns over 512-deep k
 //     blocks; each k block's weight slice is widened to fp32 once and reused by the tile's
-//     eight 12-row panels. Every output element's k order is fixed, so results do not depend
+//     twelve 12-row panels. Every output element's k order is fixed, so results do not depend
 //     on how tiles fall to threads. The epilogues mirror the GPU's: 1/rms scaling, RoPE and
 //     the KV write for QKV; the residual add for O and down; SwiGLU for gate/up, whose rows
 //     are grouped as 64 gate rows then the 64 matching up rows so one tile holds both halves;
@@ -44,8 +44,8 @@ typedef uint32_t v4u __attribute__((vector_size(16)));
 
 constexpr int kMR = 12;   // rows of one register tile (three 4-lane vectors)
 constexpr int kNR = 8;    // columns of one register tile = weight rows of one panel
-constexpr int kKC = 256;  // k block
-constexpr int kTM = 96;   // rows of one task tile
+constexpr int kKC = 512;  // k block
+constexpr int kTM = 144;  // rows of one task tile
 constexpr int kTN = 128;  // columns of one task tile
 constexpr int kGU = 64;   // feed-forward units per gate/up tile (64 gate + 64 up columns)
 constexpr int kQB = 16;   // queries per attention task
