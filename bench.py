@@ -95,7 +95,9 @@ class ClockSampler:
     def __init__(self, gpu_id: str):
         self.gpu_id = gpu_id
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        # raw samples go to $VLA_ARTIFACT_DIR (default: artifacts/ at the repository root)
+        out = os.environ.get("VLA_ARTIFACT_DIR", os.path.join(ROOT, "artifacts"))
+        self.path = os.path.join(out, f"clocks_{os.getpid()}.csv")
 
     def start(self):
         try:

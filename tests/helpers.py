@@ -27,7 +27,8 @@ def sync(seconds: float = 60.0):
             import os
             import traceback
             msg = f"GPU work did not finish within {seconds} s; exiting\n" + "".join(traceback.format_stack())
-            out = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "gpurun_out")
+            out = os.environ.get("VLA_ARTIFACT_DIR",
+                                 os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "artifacts"))
             os.makedirs(out, exist_ok=True)
             with open(os.path.join(out, "watchdog.txt"), "a") as f:
                 f.write(msg)
