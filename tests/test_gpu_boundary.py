@@ -21,8 +21,9 @@ def _bits(t):
 def test_frames_with_overlapped_boundary_copies_and_per_frame_split(vla_lib):
     """Four 3072-token frames (6 x 448 visual + 384 text rows) through an 8-block 7B-class
     stack, double-buffered: frame f's boundary copy overlaps frame f's suffix range and
-    frame f+1's prefix. Each frame uses its own split point; the host copy of h^(k) and the
-    range output equal single-stream reference runs bit for bit."""
+    frame f+1's prefix (checked on event timestamps). Each frame uses its own split point;
+    the host copy of h^(k) and the range output equal single-stream reference runs bit for
+    bit."""
     import torch
     vla = vla_lib
     s, L, M = synth.B7, 8, 3072
@@ -61,6 +62,8 @@ def test_frames_with_overlapped_boundary_copies_and_per_frame_split(vla_lib):
             done[b].synchronize()
             np.testing.assert_array_equal(pinned[b].view(torch.int16).numpy(), ref_h[f])
 
+        ev = [{n: torch.cuda.Event(enable_timing=True) for n in ("copy0", "copy1", "suffix0", "suffix1")}
+              for _ in range(4)]
         for f in range(4):
             b = f % 2
             if f >= 2:
@@ -68,8 +71,13 @@ def test_frames_with_overlapped_boundary_copies_and_per_frame_split(vla_lib):
             vla.vla_kv_reset(kvs[b], main)
             vla.vla_prefix_prefill(m.handle, xs[f], M, 0, ks[f], kvs[b], hdev[b], main)
             ready[b].record(main)
-            vla.vla_boundary_to_host(hdev[b], M, s.hidden, pinned[b], side, ready[b], done[b])
+            side.wait_event(ready[b])
+            ev[f]["copy0"].record(side)
+            vla.vla_boundary_to_host(hdev[b], M, s.hidden, pinned[b], side, None, done[b])
+            ev[f]["copy1"].record(side)
+            ev[f]["suffix0"].record(main)
             vla.vla_prefix_prefill(m.handle, hdev[b], M, ks[f], L, kvs[b], ydev[b], main)
+            ev[f]["suffix1"].record(main)
             main.wait_event(done[b])  # hdev[b] is rewritten two frames later
             if f >= 2:
                 sync(120)
@@ -78,6 +86,11 @@ def test_frames_with_overlapped_boundary_copies_and_per_frame_split(vla_lib):
         check(3)
         sync(120)
         np.testing.assert_array_equal(_bits(ydev[1]), ref_y[3])
+        # each frame's boundary copy ran while its suffix range was running (event timestamps:
+        # the copy started before the suffix ended and finished after the suffix started)
+        for f in range(4):
+            assert ev[f]["copy0"].elapsed_time(ev[f]["suffix1"]) > 0, f
+            assert ev[f]["suffix0"].elapsed_time(ev[f]["copy1"]) > 0, f
         assert vla.vla_last_async_error(m.handle) == 0
         for kv in kvs + [kv_ref]:
             vla.vla_kv_destroy(kv)
