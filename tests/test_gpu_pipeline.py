@@ -152,3 +152,39 @@ def test_7b_pipeline_overlaps_gpu_prefix_with_cpu_suffix(vla_lib):
     finally:
         vla.vla_cpu_model_destroy(cpu)
         m.close()
+
+
+def test_scheduler_drives_the_split_of_the_pipeline(vla_lib):
+    """Phi (Sec. IV-D) on the live pipeline: from observed stage times it moves the boundary
+    one block per frame toward the cheaper side, here the GPU (a tiny block costs the host
+    cores far more than the GPU), and stops at the zone's end; every frame stays correct."""
+    vla = vla_lib
+    import torch
+    s, L, M, max_ctx = synth.TINY, 3, 64, 64
+    m = Model(s, L, 8, max_ctx)
+    cpu = vla.vla_cpu_model_create(vla_cfg(s, max_ctx), m.bits[1:], 1, 2)
+    sched = vla.vla_scheduler_create(L, 1, L, 1, max_step=1, alpha=1.0)
+    try:
+        xs = [to_dev(synth.hidden_states(M, s.hidden, 80 + f)) for f in range(5)]
+        stream = torch.cuda.current_stream()
+        pl = vla.vla_pipeline_create(m.handle, cpu, M, 1)  # depth 1: each split sees the last frame
+        splits = []
+        try:
+            for f in range(5):
+                k = vla.vla_scheduler_next(sched)
+                splits.append(k)
+                vla.vla_pipeline_submit(pl, f, xs[f], M, k, stream)
+                y = np.empty((M, s.hidden), dtype=np.uint16)
+                fid, t = vla.vla_pipeline_collect(pl, y, 120000)
+                assert fid == f
+                vla.vla_scheduler_observe(sched, t)
+                np.testing.assert_array_equal(y, _composed(vla, m, cpu, xs[f], M, k, L, max_ctx))
+        finally:
+            vla.vla_pipeline_destroy(pl)
+        assert splits == [1, 2, 3, 3, 3], splits  # no move before the first observation
+        g_ms, c_ms, _ = vla.vla_scheduler_estimates(sched)
+        assert 0 < g_ms < c_ms
+    finally:
+        vla.vla_scheduler_destroy(sched)
+        vla.vla_cpu_model_destroy(cpu)
+        m.close()
