@@ -82,17 +82,14 @@ inline float hsum(v4f v) { return (v[0] + v[1]) + (v[2] + v[3]); }
 class Pool {
   public:
     explicit Pool(int n) : n_(n < 1 ? 1 : n) {
-        for (int i = 1; i < n_; ++i) th_.emplace_back([this, i] { worker(i); });
-    }
-    ~Pool() {
-        {
-            std::lock_guard<std::mutex> lk(m_);
-            stop_ = true;
-            ++gen_;
+        try {
+            for (int i = 1; i < n_; ++i) th_.emplace_back([this, i] { worker(i); });
+        } catch (...) {
+            shutdown();  // join the threads already started before the failure propagates
+            throw;
         }
-        cv_.notify_all();
-        for (auto& t : th_) t.join();
     }
+    ~Pool() { shutdown(); }
     int size() const { return n_; }
     // fn(task, thread) for every task in [0, n_tasks); returns when all have finished.
     void run(int n_tasks, const std::function<void(int, int)>& fn) {
@@ -116,6 +113,17 @@ class Pool {
     }
 
   private:
+    void shutdown() {
+        {
+            std::lock_guard<std::mutex> lk(m_);
+            stop_ = true;
+            ++gen_;
+        }
+        cv_.notify_all();
+        for (auto& t : th_)
+            if (t.joinable()) t.join();
+        th_.clear();
+    }
     void drain(int tid) {
         for (int t = next_.fetch_add(1); t < tasks_; t = next_.fetch_add(1)) (*fn_)(t, tid);
     }
