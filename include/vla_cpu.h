@@ -105,7 +105,8 @@ typedef struct {
  * suffixes in submission order on the CPU model's pool. The device current at this call
  * must be current for every later call, all frames must be submitted on one stream (the GPU
  * cache is reused frame after frame in that stream's order), and the models must outlive
- * the pipeline.
+ * the pipeline. Submit and collect may run on two different threads, but each from one
+ * thread at a time (one producer, one consumer).
  * Errors: INVALID_ARG, SHAPE (configs differ, max_tokens), RANGE (layer ranges), OOM, CUDA. */
 vla_status vla_pipeline_create(vla_prefix* gpu, vla_cpu_model* cpu, int max_tokens, int depth, vla_pipeline** out);
 
