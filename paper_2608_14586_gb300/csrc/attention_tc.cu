@@ -458,13 +458,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int DH>
 cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t stream, bool pdl) {
     using C = AttnCfg<DH>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e =
-            cudaFuncSetAttribute(attn_prefill_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    // once per process (thread-safe initialisation of local statics)
+    static const cudaError_t attr =
+        cudaFuncSetAttribute(attn_prefill_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (attr != cudaSuccess) return attr;
     const int ctx = p.pos0 + p.M;
     CUtensorMap tq, tk, tv;
     if (!make_tmap_bf16(&tq, p.q, p.M, (uint64_t)p.H * DH, p.ld_q, 128) ||
@@ -482,13 +479,12 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
     a.out = p.out;
     a.status = status;
     // persistent: one CTA per SM (tensor-memory kernels get one per SM), each walking its pairs
-    static int sms = 0;
-    if (!sms) {
-        int dev = 0;
+    static const int sms = [] {
+        int dev = 0, n = 0;
         cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-    }
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        return n > 0 ? n : 1;
+    }();
     const int units = ((p.M + 2 * kBM - 1) / (2 * kBM)) * p.H;
     const dim3 grid(units < sms ? units : sms);
     return launch_ex(attn_prefill_tc_kernel<DH>, grid, dim3(kThreads), C::SMEM, stream, pdl, tq, tk, tv, a);

@@ -338,14 +338,9 @@ cudaError_t prepare(int cs, size_t smem) {
 template <int G>
 cudaError_t launch(const DecKVMaps& maps, const AttnDecTcParams& p, cudaStream_t s, bool pdl) {
     const size_t smem = smem_layout(p.rows).total;
-    static size_t attr_smem = 0;
-    static int attr_cs = 0;
-    if (smem > attr_smem || p.cs > attr_cs) {
-        cudaError_t e = prepare<G>(p.cs, smem);
-        if (e != cudaSuccess) return e;
-        attr_smem = smem > attr_smem ? smem : attr_smem;
-        attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
-    }
+    static KernelAttrCache attrs;
+    const cudaError_t ea = attrs.ensure(smem, p.cs, [](int cs, size_t sm) { return prepare<G>(cs, sm); });
+    if (ea != cudaSuccess) return ea;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(p.cs, p.Hkv, p.nb);
     cfg.blockDim = dim3(kThreads);

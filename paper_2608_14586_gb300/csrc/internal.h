@@ -6,9 +6,33 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 namespace vla {
 
 using bf16 = __nv_bfloat16;
+
+// Launch attributes of one kernel, raised on demand: the dynamic shared-memory limit and the
+// cluster size `set(cs, smem)` has been asked for only ever grow, under a lock, so host
+// threads may launch concurrently. The library drives one device per process.
+struct KernelAttrCache {
+    std::mutex mu;
+    size_t smem = 0;
+    int cs = 0;
+    template <class Set>
+    cudaError_t ensure(size_t need_smem, int need_cs, Set&& set) {
+        std::lock_guard<std::mutex> lk(mu);
+        if (need_smem <= smem && need_cs <= cs) return cudaSuccess;
+        const size_t s = need_smem > smem ? need_smem : smem;
+        const int c = need_cs > cs ? need_cs : cs;
+        const cudaError_t e = set(c, s);
+        if (e == cudaSuccess) {
+            smem = s;
+            cs = c;
+        }
+        return e;
+    }
+};
 
 // ---------------------------------------------------------------------------------------
 // tcgen05 GEMM: C[M,N] = A[M,K] * B[N,K]^T with a fused epilogue

@@ -858,8 +858,7 @@ vla_status vla_op_gemm_bf16(const void* A, const void* B, int M, int N, int K, v
     ep.N = N;
     ep.out = (bf16*)C;
     ep.ld_out = N;
-    static int sms = 0;
-    if (!sms) sms = vla::device_sm_count();
+    static const int sms = vla::device_sm_count();
     return cuda_status(vla::launch_gemm(vla::kEpiPlain, kBN, ta, tb, M, N, K, ep, sms, (cudaStream_t)stream));
 }
 
