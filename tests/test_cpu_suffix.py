@@ -119,6 +119,43 @@ def test_gqa_7b_block_ragged_tokens_match_oracle(vla):
         m.close()
 
 
+@pytest.mark.parametrize("shape", [
+    # 2 query heads per KV head, head_dim 64, FFN 700 (padded to 704: a partial gate/up unit)
+    synth.ModelShape(hidden=256, n_heads=8, n_kv_heads=4, head_dim=64, ffn=700),
+    # 8 query heads per KV head, head_dim 128, FFN 520 (padded to 576)
+    synth.ModelShape(hidden=512, n_heads=16, n_kv_heads=2, head_dim=128, ffn=520),
+], ids=["gqa2_dh64", "gqa8_dh128"])
+def test_other_head_groupings_match_oracle(vla, shape):
+    """The other supported query-per-KV-head groupings and an FFN width that is not a
+    multiple of the gate/up unit: two blocks over 29 tokens, then two decode steps."""
+    s, L, M, max_ctx = shape, 2, 29, 40
+    m = CpuModel(vla, s, L, 13, max_ctx, gain="random", n_threads=3)
+    try:
+        xb = synth.hidden_states(M, s.hidden, 13)
+        cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, max_ctx)
+        per_block = []
+        ref = oracle.prefix_forward(_f64(xb), m.w64, 0, L, cache, s, per_block=per_block)
+        kv = vla.vla_cpu_kv_create(m.h, 0, L, max_ctx)
+        h = m.run(xb, 0, 1, kv)
+        assert rel_l2(_f64(h), per_block[0]) < REL_L2_BLOCK
+        y = m.run(h, 1, L, kv)
+        assert rel_l2(_f64(y), ref) < REL_L2_BLOCK
+        assert cos_sim(_f64(y), ref) > COS_FINAL
+        for l in range(L):
+            k, v = m.kv_planes(kv, l, max_ctx, M)
+            assert rel_l2(k, cache.k[l][:, :M]) < REL_L2_BLOCK
+            assert rel_l2(v, cache.v[l][:, :M]) < REL_L2_BLOCK
+        for t in range(2):
+            xt = synth.decode_hidden(t, s.hidden, 13)
+            yt = m.run(xt, 0, L, kv)
+            rt = oracle.decode_step(_f64(xt), m.w64, 0, L, cache, s)
+            assert rel_l2(_f64(yt), rt) < REL_L2_BLOCK
+        assert vla.vla_cpu_kv_length(kv) == M + 2
+        vla.vla_cpu_kv_destroy(kv)
+    finally:
+        m.close()
+
+
 def _cache_with_context(vla, m, s, max_ctx, kb, vb):
     """A host cache whose positions [0, p0) hold the given K/V bits: a p0-token prefill sets
     the length, then its K/V rows are overwritten with the given ones."""
@@ -224,6 +261,18 @@ def test_model_over_a_suffix_range_and_argument_errors(vla):
         assert lib.vla_pipeline_destroy(None) == 0 and lib.vla_pipeline_in_flight(None) == -1
         assert lib.vla_pipeline_collect(None, None, None, 0, None) == 1
         assert lib.vla_status_str(10) == b"all pipeline slots in flight"
+        w1 = [synth.layer_weights(s, 2, 0)]
+        for bad in (dict(head_dim=96),                     # head_dim other than 64 / 128
+                    dict(n_heads=6, n_kv_heads=4),         # query heads not a multiple of KV heads
+                    dict(n_heads=12, n_kv_heads=4),        # 3 query heads per KV head
+                    dict(hidden=320)):                     # hidden not a multiple of 256
+            c = _cfg(vla, s, max_ctx)
+            for k, v in bad.items():
+                setattr(c, k, v)
+            assert status(vla.vla_cpu_model_create, c, w1, 0) == "VLA_ERR_UNSUPPORTED", bad
+        c = _cfg(vla, s, max_ctx)
+        c.rope_base = 1.0
+        assert status(vla.vla_cpu_model_create, c, w1, 0) == "VLA_ERR_INVALID_ARG"
         vla.vla_cpu_kv_destroy(kv)
     finally:
         m.close()
