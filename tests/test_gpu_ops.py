@@ -41,6 +41,8 @@ def test_gemm_matches_definition(vla_lib, M, N, K):
     (200, 32, 8, 128, 0),     # ragged M, GQA group 4
     (130, 8, 2, 128, 77),     # continuing context
     (1, 4, 1, 64, 5),         # one query, MQA
+    (96, 8, 4, 64, 3),        # GQA group 2
+    (150, 16, 2, 128, 9),     # GQA group 8, ragged M, continuing context
     (1024, 32, 8, 128, 0),    # 7B shape
 ])
 def test_attention_prefill_matches_oracle(vla_lib, M, H, Hkv, dh, pos0):

@@ -171,3 +171,50 @@ def test_decode_7b_two_blocks_random_context(vla_lib):
         vla.vla_kv_destroy(kv)
     finally:
         m.close()
+
+
+@pytest.mark.parametrize("shape", [
+    # 2 query heads per KV head, head_dim 64, FFN 700 (zero-padded to the gate/up unit)
+    synth.ModelShape(hidden=256, n_heads=8, n_kv_heads=4, head_dim=64, ffn=700),
+    # 8 query heads per KV head, head_dim 128, FFN 520
+    synth.ModelShape(hidden=512, n_heads=16, n_kv_heads=2, head_dim=128, ffn=520),
+], ids=["gqa2_dh64", "gqa8_dh128"])
+def test_other_head_groupings_prefill_and_decode(vla_lib, shape):
+    """The other supported query-per-KV-head groupings: two blocks over 29 tokens (block by
+    block against the oracle, with the written cache), then three decode steps."""
+    import torch
+    vla = vla_lib
+    s, L, M, max_ctx = shape, 2, 29, 40
+    m = Model(s, L, 13, max_ctx, gain="random")
+    try:
+        xb = synth.hidden_states(M, s.hidden, 13)
+        cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, max_ctx)
+        per_block = []
+        ref = oracle.prefix_forward(oracle.bf16_to_f64(xb), m.weights64(), 0, L, cache, s, per_block=per_block)
+        kv = vla.vla_kv_create(m.handle, 0, L, max_ctx)
+        x = to_dev(xb)
+        h = torch.empty_like(x)
+        vla.vla_prefix_prefill(m.handle, x, M, 0, 1, kv, h)
+        y = torch.empty_like(x)
+        vla.vla_prefix_prefill(m.handle, h, M, 1, L, kv, y)
+        sync()
+        assert vla.vla_last_async_error(m.handle) == 0
+        assert rel_l2(from_dev(h), per_block[0]) < REL_L2_BLOCK
+        assert rel_l2(from_dev(y), ref) < REL_L2_BLOCK
+        assert cos_sim(from_dev(y), ref) > COS_FINAL
+        for l in range(L):
+            K, V = _kv_planes(vla, kv, l, s, max_ctx, M)
+            assert rel_l2(K, cache.k[l][:, :M]) < REL_L2_BLOCK
+            assert rel_l2(V, cache.v[l][:, :M]) < REL_L2_BLOCK
+        out = torch.empty((1, s.hidden), dtype=torch.bfloat16, device="cuda")
+        for t in range(3):
+            xt = synth.decode_hidden(t, s.hidden, 13)
+            rt = oracle.decode_step(oracle.bf16_to_f64(xt), m.weights64(), 0, L, cache, s)
+            vla.vla_prefix_decode(m.handle, to_dev(xt), 0, L, kv, out)
+            sync()
+            assert rel_l2(from_dev(out), rt) < REL_L2_BLOCK, t
+        assert vla.vla_kv_length(kv) == M + 3
+        assert vla.vla_last_async_error(m.handle) == 0
+        vla.vla_kv_destroy(kv)
+    finally:
+        m.close()
