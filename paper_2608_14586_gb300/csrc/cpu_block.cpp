@@ -50,6 +50,7 @@ constexpr int kTN = 128;  // columns of one task tile
 constexpr int kGU = 64;   // feed-forward units per gate/up tile (64 gate + 64 up columns)
 constexpr int kQB = 16;   // queries per attention task
 constexpr int kKB = 64;   // keys per attention block
+constexpr int kKPan = (kKB + kMR - 1) / kMR;  // register-tile panels of one key block
 
 inline float bf2f(uint16_t b) {
     const uint32_t u = (uint32_t)b << 16;
@@ -163,7 +164,7 @@ struct Scratch {
     std::vector<float> apack;   // [kTM / kMR][kKC][kMR]
     std::vector<float> bf;      // [kKC][kNR]: one panel's k block widened to fp32
     std::vector<float> ctile;   // [kTN][kTM], column-major
-    std::vector<float> qpk, kpk, vpk, ppk, st, ot;  // attention operands (see attention())
+    std::vector<float> qpk, ppk, st, ot;  // attention operands (see attention())
     std::vector<float> mx, l;                        // [G * kQB]
 };
 
@@ -218,6 +219,7 @@ struct vla_cpu_model {
     std::vector<uint16_t> h[2], q, att, xmid, mbuf;
     std::vector<float> rinv;
     std::vector<float> xrows;  // [4][max K]: the rows of a short (decode) projection in fp32
+    std::vector<float> kvpk;   // one call's keys and values as register-tile panels (attention())
     ~vla_cpu_model() { delete pool; }
 };
 
@@ -365,25 +367,49 @@ void row_rinv(Model* m, const uint16_t* x, int M, float* out) {
 }
 
 // Causal GQA attention of M queries at positions p0.. over cache positions [0, p0 + M).
-// Per task (KV head g, block of kQB queries): the G query heads' vectors of the block form
-// nq = G * rows columns. Per 64-key block: S^T = K Q^T and O^T += V^T P^T on the register
-// tile (keys resp. head dims as rows, queries as columns), with the online-softmax update
-// (running max, rescale of the running sum and output) in between. Keys past a query's
-// position get probability 0 and a block wholly past it leaves its state unchanged.
+// Every 64-key block of every KV head is first widened to fp32 register-tile panels, once
+// per call. Per task (KV head g, block of kQB queries): the G query heads' vectors of the
+// block form nq = G * rows columns. Per 64-key block: S^T = K Q^T and O^T += V^T P^T on the
+// register tile (keys resp. head dims as rows, queries as columns), with the online-softmax
+// update (running max, rescale of the running sum and output) in between. Keys past a
+// query's position get probability 0 and a block wholly past it leaves its state unchanged.
 void attention(Model* m, const uint16_t* q, const uint16_t* kp, const uint16_t* vp, int max_ctx, int p0, int M,
                uint16_t* out) {
     const int H = m->cfg.n_heads, Hkv = m->cfg.n_kv_heads, dh = m->cfg.head_dim, G = H / Hkv;
     const float scale = 1.0f / std::sqrt((float)dh);
     const int nqb = (M + kQB - 1) / kQB;
     const int dpan = (dh + kMR - 1) / kMR;  // head-dim panels of the O tile
+    // per (g, key block): keys [kKPan][dh][kMR] (zero rows past the context), then values
+    // [dpan][kKB][kMR]
+    const int nkb = (p0 + M + kKB - 1) / kKB;
+    const size_t kstride = (size_t)kKPan * dh * kMR, bstride = kstride + (size_t)dpan * kKB * kMR;
+    float* kvpk = m->kvpk.data();
+    m->pool->run(Hkv * nkb, [&](int t, int) {
+        const int g = t % Hkv, kb = t / Hkv, kb0 = kb * kKB, kn = std::min(kKB, p0 + M - kb0);
+        float* kpk = kvpk + ((size_t)g * nkb + kb) * bstride;
+        float* vpk = kpk + kstride;
+        const uint16_t* kg = kp + (size_t)g * max_ctx * dh;
+        const uint16_t* vg = vp + (size_t)g * max_ctx * dh;
+        for (int j = 0; j < (kn + kMR - 1) / kMR * kMR; ++j) {
+            float* dst = kpk + (size_t)(j / kMR) * dh * kMR + (j % kMR);
+            if (j < kn) {
+                const uint16_t* src = kg + (size_t)(kb0 + j) * dh;
+                for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = bf2f(src[d]);
+            } else {
+                for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = 0.f;
+            }
+        }
+        for (int j = 0; j < kn; ++j) {
+            const uint16_t* src = vg + (size_t)(kb0 + j) * dh;
+            for (int d = 0; d < dh; ++d) vpk[((size_t)(d / kMR) * kKB + j) * kMR + (d % kMR)] = bf2f(src[d]);
+        }
+    });
     m->pool->run(Hkv * nqb, [&](int t, int tid) {
         Scratch& s = m->scratch[tid];
         const int g = t % Hkv, qb = nqb - 1 - t / Hkv;  // longest query blocks first
         const int r0 = qb * kQB, r1 = std::min(M, r0 + kQB), nr = r1 - r0;
         const int nq = G * nr, nqp = (nq + kNR - 1) / kNR;  // query columns, column panels
         float* qpk = s.qpk.data();  // [nqp][dh][kNR]   queries (scaled), B operand of S
-        float* kpk = s.kpk.data();  // [6][dh][kMR]     keys of the block, A operand of S
-        float* vpk = s.vpk.data();  // [dpan][kKB][kMR] values of the block, A operand of O
         float* ppk = s.ppk.data();  // [nqp][kKB][kNR]  probabilities, B operand of O
         float* st = s.st.data();    // [nqp * kNR][kKB] scores, query-major
         float* ot = s.ot.data();    // [nqp * kNR][dh]  unnormalised outputs, query-major
@@ -398,24 +424,11 @@ void attention(Model* m, const uint16_t* q, const uint16_t* kp, const uint16_t* 
         std::fill(s.mx.begin(), s.mx.begin() + nq, -INFINITY);
         std::fill(s.l.begin(), s.l.begin() + nq, 0.f);
         const int nkeys = p0 + r1;  // keys visible to the block's last query
-        const uint16_t* kg = kp + (size_t)g * max_ctx * dh;
-        const uint16_t* vg = vp + (size_t)g * max_ctx * dh;
         for (int kb0 = 0; kb0 < nkeys; kb0 += kKB) {
             const int kn = std::min(kKB, nkeys - kb0);
             const int kpan = (kn + kMR - 1) / kMR;
-            for (int j = 0; j < kpan * kMR; ++j) {
-                float* dst = kpk + (size_t)(j / kMR) * dh * kMR + (j % kMR);
-                if (j < kn) {
-                    const uint16_t* src = kg + (size_t)(kb0 + j) * dh;
-                    for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = bf2f(src[d]);
-                } else {
-                    for (int d = 0; d < dh; ++d) dst[(size_t)d * kMR] = 0.f;
-                }
-            }
-            for (int j = 0; j < kn; ++j) {
-                const uint16_t* src = vg + (size_t)(kb0 + j) * dh;
-                for (int d = 0; d < dh; ++d) vpk[((size_t)(d / kMR) * kKB + j) * kMR + (d % kMR)] = bf2f(src[d]);
-            }
+            const float* kpk = kvpk + ((size_t)g * nkb + kb0 / kKB) * bstride;
+            const float* vpk = kpk + kstride;
             for (int cp = 0; cp < nqp; ++cp)
                 for (int kq = 0; kq < kpan; ++kq)
                     micro_any(kn - kq * kMR, kpk + (size_t)kq * dh * kMR, qpk + (size_t)cp * dh * kNR, dh,
@@ -583,10 +596,7 @@ vla_status vla_cpu_model_create(const vla_config* cfg, const vla_layer_weights* 
             s.bf.assign((size_t)kKC * kNR, 0.f);
             s.ctile.assign((size_t)kTM * kTN, 0.f);
             const int qcols = (G * kQB + kNR - 1) / kNR * kNR;
-            const int dpan = (dh + kMR - 1) / kMR, kpan = (kKB + kMR - 1) / kMR;
             s.qpk.assign((size_t)qcols * dh, 0.f);
-            s.kpk.assign((size_t)kpan * dh * kMR, 0.f);
-            s.vpk.assign((size_t)dpan * kKB * kMR, 0.f);
             s.ppk.assign((size_t)qcols * kKB, 0.f);
             s.st.assign((size_t)qcols * kKB, 0.f);
             s.ot.assign((size_t)qcols * dh, 0.f);
@@ -649,6 +659,8 @@ vla_status vla_cpu_model_create(const vla_config* cfg, const vla_layer_weights* 
         m->mbuf.resize((size_t)T * m->F_pad);
         m->rinv.resize(T);
         m->xrows.resize((size_t)kGemvRows * std::max(std::max(D, m->qc), m->F_pad));
+        const size_t kv_blocks = (size_t)Hkv * ((T + kKB - 1) / kKB);
+        m->kvpk.assign(kv_blocks * ((size_t)kKPan * dh * kMR + (size_t)((dh + kMR - 1) / kMR) * kKB * kMR), 0.f);
     } catch (const std::bad_alloc&) {
         delete m;
         return VLA_ERR_OOM;
