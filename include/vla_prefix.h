@@ -24,9 +24,9 @@
  *     are detected on the host and returned before anything is enqueued. A kernel whose
  *     bounded wait runs out records a device status read by vla_last_async_error.
  *   - No C++ exception crosses the ABI. No call takes ownership of caller memory.
- *   - Threads: calls on one vla_prefix (and on the vla_kv objects made from it) must not
- *     overlap; separate objects may be driven from separate host threads. One device per
- *     process.
+ *   - Threads: drive the library from one host thread at a time (calls must not overlap;
+ *     some launch paths cache kernel attributes per process without a lock). One device
+ *     per process.
  */
 #ifndef VLA_PREFIX_H
 #define VLA_PREFIX_H

@@ -521,9 +521,14 @@ cudaError_t attn_dec_prepare(int cs, size_t smem) {
 template <int DH, int G>
 cudaError_t launch_attn_dec(const AttnDecParams& p, cudaStream_t s, bool pdl) {
     const size_t smem = attn_dec_smem<DH, G>(p);
-    static KernelAttrCache attrs;
-    const cudaError_t ea = attrs.ensure(smem, p.cs, [](int cs, size_t sm) { return attn_dec_prepare<DH, G>(cs, sm); });
-    if (ea != cudaSuccess) return ea;
+    static size_t attr_smem = 0;
+    static int attr_cs = 0;
+    if (smem > attr_smem || p.cs > attr_cs) {
+        cudaError_t e = attn_dec_prepare<DH, G>(p.cs, smem);
+        if (e != cudaSuccess) return e;
+        attr_smem = smem > attr_smem ? smem : attr_smem;
+        attr_cs = p.cs > attr_cs ? p.cs : attr_cs;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(p.cs, p.Hkv, p.nb);
     cfg.blockDim = dim3(kAttnThreads);

@@ -442,11 +442,13 @@ template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K, const EpiParams& ep,
                        int num_sms, cudaStream_t stream, bool pdl) {
     using C = GemmCfg<BN>;
+    static bool attr_set = false;
     auto kern = gemm_bf16_tcgen05<BN, EPI>;
-    // once per process (thread-safe initialisation of a local static)
-    static const cudaError_t attr = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                         C::SMEM_BYTES);
-    if (attr != cudaSuccess) return attr;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
     const int tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
     const int grid = tiles < num_sms ? tiles : num_sms;
     return launch_ex(kern, dim3(grid), dim3(kThreads), C::SMEM_BYTES, stream, pdl, A, B, M, N, K, ep);
