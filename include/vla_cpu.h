@@ -13,9 +13,10 @@
  * folded into the weights and rounded to bf16 the same way); products accumulate in fp32;
  * the stage outputs the GPU stores as bf16 (q, k, v, the attention output, the mid-block
  * residual, the SwiGLU product, the block output) are rounded to bf16 at the same points.
- * Results do not depend on the thread count. Softmax, SiLU and the rotary angles use the C
- * library's exp / sin / cos (angles in double), so CPU and GPU agree to rounding, not bit
- * for bit.
+ * Results do not depend on the thread count. Softmax and SiLU use a portable four-lane exp
+ * (Cody-Waite argument reduction and a degree-7 Taylor polynomial: within 2 ulp over the
+ * normal fp32 range, results below it flushed to 0); the rotary angles use the C library's
+ * sin / cos in double. CPU and GPU agree to rounding, not bit for bit.
  *
  * Conventions: tensors are bf16 (uint16 bit patterns), row-major, contiguous, in ordinary
  * host memory unless stated. Layer indices are absolute (block l of the model). No call

@@ -34,6 +34,7 @@
 #include <thread>
 #include <vector>
 
+#include "cpu_math.h"
 #include "vla_cpu.h"
 
 namespace {
@@ -51,6 +52,7 @@ constexpr int kGU = 64;   // feed-forward units per gate/up tile (64 gate + 64 u
 constexpr int kQB = 16;   // queries per attention task
 constexpr int kKB = 64;   // keys per attention block
 constexpr int kKPan = (kKB + kMR - 1) / kMR;  // register-tile panels of one key block
+static_assert(kKB % 4 == 0 && kGU % 4 == 0, "the softmax and SiLU loops take four lanes at a time");
 
 inline float bf2f(uint16_t b) {
     const uint32_t u = (uint32_t)b << 16;
@@ -442,13 +444,21 @@ void attention(Model* m, const uint16_t* q, const uint16_t* kp, const uint16_t* 
                 float smax = -INFINITY;
                 for (int j = 0; j < jn; ++j) smax = std::max(smax, sc[j]);
                 const float mold = s.mx[c], mnew = std::max(mold, smax);
-                const float corr = std::exp(mold - mnew);  // 0 when mold = -inf
+                const float corr = vla_cpu::exp1(mold - mnew);  // 0 when mold = -inf
                 float lsum = s.l[c] * corr;
                 float* pc = ppk + (size_t)(c / kNR) * kKB * kNR + (c % kNR);
+                // four scores at a time (the lanes past jn read scores of this block's
+                // zero-padded key rows and are dropped), then summed in key order
+                float pv[kKB];
+                for (int j = 0; j < jn; j += 4) {
+                    v4f a;
+                    std::memcpy(&a, sc + j, sizeof a);
+                    const v4f e = vla_cpu::exp4(a - mnew);
+                    std::memcpy(pv + j, &e, sizeof e);
+                }
                 for (int j = 0; j < jn; ++j) {
-                    const float pj = std::exp(sc[j] - mnew);
-                    lsum += pj;
-                    pc[(size_t)j * kNR] = pj;
+                    lsum += pv[j];
+                    pc[(size_t)j * kNR] = pv[j];
                 }
                 float* oc = ot + (size_t)c * dh;
                 for (int d = 0; d < dh; ++d) oc[d] *= corr;
@@ -528,9 +538,14 @@ void block(Model* m, int l, const uint16_t* x, int M, int p0, vla_cpu_kv* kv, ui
         for (int r = 0; r < rows; ++r) {
             const float ri = rinv[m0 + r];
             uint16_t* dst = mb + (size_t)(m0 + r) * F_pad + u0;
-            for (int i = 0; i < kGU; ++i) {
-                const float gt = C[(size_t)i * ldc + r] * ri, up = C[(size_t)(kGU + i) * ldc + r] * ri;
-                dst[i] = f2bf(gt / (1.0f + std::exp(-gt)) * up);
+            for (int i = 0; i < kGU; i += 4) {
+                v4f gt, up;
+                for (int e = 0; e < 4; ++e) {
+                    gt[e] = C[(size_t)(i + e) * ldc + r] * ri;
+                    up[e] = C[(size_t)(kGU + i + e) * ldc + r] * ri;
+                }
+                const v4f sw = gt / (1.0f + vla_cpu::exp4(-gt)) * up;
+                for (int e = 0; e < 4; ++e) dst[i + e] = f2bf(sw[e]);
             }
         }
     });
