@@ -11,8 +11,9 @@
 //     of a k step (24 fp32 vector accumulators; GCC vector extensions over 128-bit lanes: NEON
 //     on an Arm host, SSE on x86). A task tile is 144 rows x 128 columns over 512-deep k
 //     blocks; each k block's weight slice is widened to fp32 once and reused by the tile's
-//     twelve 12-row panels. Every output element's k order is fixed, so results do not depend
-//     on how tiles fall to threads. The epilogues mirror the GPU's: 1/rms scaling, RoPE and
+//     twelve 12-row panels, and a task takes two column tiles so that each packed A block
+//     serves both. Every output element's k order is fixed, so results do not depend on how
+//     tiles fall to threads. The epilogues mirror the GPU's: 1/rms scaling, RoPE and
 //     the KV write for QKV; the residual add for O and down; SwiGLU for gate/up, whose rows
 //     are grouped as 64 gate rows then the 64 matching up rows so one tile holds both halves;
 //   * attention: one task per (KV head, block of 16 queries), longest first; per 64-key block
@@ -48,6 +49,7 @@ constexpr int kNR = 8;    // columns of one register tile = weight rows of one p
 constexpr int kKC = 512;  // k block
 constexpr int kTM = 144;  // rows of one task tile
 constexpr int kTN = 128;  // columns of one task tile
+constexpr int kTG = 2;    // column tiles per task at most (they share one packed A block)
 constexpr int kGU = 64;   // feed-forward units per gate/up tile (64 gate + 64 up columns)
 constexpr int kQB = 16;   // queries per attention task
 constexpr int kKB = 64;   // keys per attention block
@@ -165,7 +167,7 @@ struct Packed {
 struct Scratch {
     std::vector<float> apack;   // [kTM / kMR][kKC][kMR]
     std::vector<float> bf;      // [kKC][kNR]: one panel's k block widened to fp32
-    std::vector<float> ctile;   // [kTN][kTM], column-major
+    std::vector<float> ctile;   // kTG tiles of [kTN][kTM], column-major
     std::vector<float> qpk, ppk, st, ot;  // attention operands (see attention())
     std::vector<float> mx, l;                        // [G * kQB]
 };
@@ -314,13 +316,17 @@ void gemm(Model* m, const uint16_t* A, int M, const Packed& B, const Epi& epi) {
         });
         return;
     }
+    // A task is one block of kTM rows times up to kTG column tiles, which reuse each packed
+    // A block; fewer column tiles per task where that would leave under 4 tasks per thread.
     const int tm = (M + kTM - 1) / kTM, tn = B.N / kTN;
-    m->pool->run(tm * tn, [&](int t, int tid) {
+    int grp = kTG;
+    while (grp > 1 && tm * ((tn + grp - 1) / grp) < 4 * m->pool->size()) grp >>= 1;
+    const int tg = (tn + grp - 1) / grp;
+    m->pool->run(tm * tg, [&](int t, int tid) {
         Scratch& s = m->scratch[tid];
-        const int im = t % tm, in = t / tm;
-        const int m0 = im * kTM, rows = std::min(kTM, M - m0), n0 = in * kTN;
+        const int im = t % tm, j0 = (t / tm) * grp, j1 = std::min(tn, j0 + grp);
+        const int m0 = im * kTM, rows = std::min(kTM, M - m0);
         const int np = (rows + kMR - 1) / kMR;
-        float* C = s.ctile.data();
         float* bf = s.bf.data();
         for (int k0 = 0; k0 < K; k0 += kKC) {
             const int kc = std::min(kKC, K - k0);
@@ -336,18 +342,21 @@ void gemm(Model* m, const uint16_t* A, int M, const Packed& B, const Epi& epi) {
                     }
                 }
             }
-            for (int j = 0; j < kTN / kNR; ++j) {
-                const uint16_t* bp = B.w.data() + ((size_t)(n0 / kNR + j) * K + k0) * kNR;
-                for (int e = 0; e < kc * kNR; e += 4) {
-                    const v4f v = ld_bf4(bp + e);
-                    std::memcpy(bf + e, &v, sizeof v);
+            for (int jt = j0; jt < j1; ++jt) {
+                float* C = s.ctile.data() + (size_t)(jt - j0) * kTN * kTM;
+                for (int j = 0; j < kTN / kNR; ++j) {
+                    const uint16_t* bp = B.w.data() + ((size_t)(jt * kTN / kNR + j) * K + k0) * kNR;
+                    for (int e = 0; e < kc * kNR; e += 4) {
+                        const v4f v = ld_bf4(bp + e);
+                        std::memcpy(bf + e, &v, sizeof v);
+                    }
+                    for (int p = 0; p < np; ++p)
+                        micro_any(rows - p * kMR, s.apack.data() + (size_t)p * kKC * kMR, bf, kc,
+                                  C + (size_t)j * kNR * kTM + p * kMR, kTM, k0 == 0);
                 }
-                for (int p = 0; p < np; ++p)
-                    micro_any(rows - p * kMR, s.apack.data() + (size_t)p * kKC * kMR, bf, kc,
-                              C + (size_t)j * kNR * kTM + p * kMR, kTM, k0 == 0);
             }
         }
-        epi(m0, rows, n0, C, kTM);
+        for (int jt = j0; jt < j1; ++jt) epi(m0, rows, jt * kTN, s.ctile.data() + (size_t)(jt - j0) * kTN * kTM, kTM);
     });
 }
 
@@ -609,7 +618,7 @@ vla_status vla_cpu_model_create(const vla_config* cfg, const vla_layer_weights* 
         for (Scratch& s : m->scratch) {
             s.apack.assign((size_t)kTM * kKC, 0.f);
             s.bf.assign((size_t)kKC * kNR, 0.f);
-            s.ctile.assign((size_t)kTM * kTN, 0.f);
+            s.ctile.assign((size_t)kTG * kTM * kTN, 0.f);
             const int qcols = (G * kQB + kNR - 1) / kNR * kNR;
             s.qpk.assign((size_t)qcols * dh, 0.f);
             s.ppk.assign((size_t)qcols * kKB, 0.f);
