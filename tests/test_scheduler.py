@@ -99,3 +99,45 @@ def test_invalid_configs(vla):
         vla.vla_scheduler_create(8, 0, 8, 4, alpha=0.0)
     assert lib.vla_scheduler_next(None, None) == -1
     assert lib.vla_scheduler_destroy(None) == 0
+
+
+def test_closed_loop_tracks_the_eq13_optimum_as_costs_change(vla):
+    """Frames simulated from true per-block costs that change mid-run (the GPU slows 8x at
+    frame 20, as under a co-tenant the controller is not told about, then recovers at frame
+    45), with 5% multiplicative noise on every stage time. Φ only sees the observed times.
+    After each change it reaches the split that minimises Eq. 13 for the new costs within a
+    bounded number of frames, stays within one block of it, never leaves the zone and never
+    moves more than max_step blocks per frame."""
+    import random
+    rng = random.Random(7)
+    N, k_min, k_max, step = 32, 12, 32, 2
+    x = 0.2
+    phases = [(0, 1.0, 24.0), (20, 8.0, 24.0), (45, 1.0, 24.0)]  # (first frame, g, c) in ms per block
+
+    def truth(t):
+        return [(g, c) for f, g, c in phases if f <= t][-1]
+
+    def best(g, c):
+        return min(range(k_min, k_max + 1), key=lambda p: (_interval(p, g, c, x, N), -p))
+
+    s = vla.vla_scheduler_create(N, k_min, k_max, 24, max_step=step, alpha=0.5)
+    try:
+        k, trace = 24, []
+        for t in range(70):
+            g, c = truth(t)
+            noise = lambda: 1.0 + rng.uniform(-0.05, 0.05)  # noqa: E731
+            f = vla.VlaFrameTimes(t_gpu_ms=k * g * noise(), t_xfer_ms=x * noise(),
+                                  t_cpu_ms=(N - k) * c * noise(), split=k, n_tokens=1)
+            vla.vla_scheduler_observe(s, f)
+            k_next = vla.vla_scheduler_next(s)
+            assert k_min <= k_next <= k_max and abs(k_next - k) <= step
+            k = k_next
+            trace.append(k)
+        assert [best(g, c) for _, g, c in phases] == [31, 24, 31]
+        for start, g, c in phases:
+            opt = best(g, c)
+            settle = start + 8  # optima 31, 24, 31: 7 blocks at 2 per frame, plus the averages' lag
+            end = next((f for f, _, _ in phases if f > start), 70)
+            assert all(abs(p - opt) <= 1 for p in trace[settle:end]), (start, opt, trace[start:end])
+    finally:
+        vla.vla_scheduler_destroy(s)
