@@ -5,6 +5,7 @@ import glob
 import os
 import re
 import shutil
+import subprocess
 
 import pytest
 
@@ -81,3 +82,30 @@ def test_binding_names_match_the_header():
     import paper_2608_14586_gb300 as vla
     for n in _declared_functions():
         assert n in vla.__all__, n
+
+
+def test_headers_are_plain_c_and_the_readme_example_compiles():
+    """Every public header compiles as C (not only C++), and the C usage example in the README
+    matches the declared signatures (wrapped in a function whose parameters supply the
+    buffers, streams and events it uses)."""
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    cuda_inc = "/usr/local/cuda/include"
+    if not os.path.exists(os.path.join(cuda_inc, "cuda_runtime.h")):
+        pytest.skip("CUDA headers not found")
+    with open(os.path.join(ROOT, "README.md")) as f:
+        readme = f.read()
+    m = re.search(r"```c\n(.*?)```", readme, flags=re.S)
+    assert m, "README has no C example"
+    body = "\n".join(line for line in m.group(1).splitlines() if not line.startswith("#include"))
+    src = ("#include <cuda_runtime.h>\n"
+           + "".join(f'#include "{os.path.basename(h)}"\n'
+                     for h in sorted(glob.glob(os.path.join(ROOT, "include", "*.h"))))
+           + "void example(const vla_layer_weights* layers, const void* h_in, void* h_out, void* pinned,\n"
+             "             const void* x1, void* y1, cudaStream_t stream, cudaStream_t side_stream,\n"
+             "             cudaEvent_t ready, cudaEvent_t done) {\n" + body + "\n}\n")
+    r = subprocess.run([cc, "-std=c11", "-fsyntax-only", "-Wall", "-Werror", "-x", "c", "-",
+                        "-I", os.path.join(ROOT, "include"), "-I", cuda_inc],
+                       input=src, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
