@@ -58,6 +58,11 @@ MUTANTS = [
      "xm = o.reshape(len(rows), H * dh) @ w.w_o.T"),
     ("rows: context keys ignored", "k_all = np.concatenate([ctx_k[:, :p0], k], axis=1)",
      "k_all = np.concatenate([np.zeros_like(ctx_k[:, :p0]), k], axis=1)"),
+    # seeding a cache with a given context
+    ("fill swaps the planes", "self.k[layer][:, :n] = k\n        self.v[layer][:, :n] = v",
+     "self.k[layer][:, :n] = v\n        self.v[layer][:, :n] = k"),
+    ("fill length off by one", "self.length[layer] = n\n", "self.length[layer] = n - 1\n"),
+    ("fill reads the head axis as length", "n = k.shape[1]", "n = k.shape[0]"),
     # layer range and boundary
     ("range reuses the first block's weights", "h = block_forward(h, weights[l], cache, l, shape)",
      "h = block_forward(h, weights[layer_begin], cache, l, shape)"),

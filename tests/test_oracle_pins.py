@@ -361,6 +361,52 @@ def test_prefill_then_decode_equals_longer_prefill():
     assert c.length == {0: 6, 1: 6}
 
 
+def test_kv_fill_seeds_context_like_a_prefill():
+    """A cache seeded by fill() with a prefill's own keys and values continues exactly like
+    the cache that prefill wrote: a decode step after it equals the longer prefill's row."""
+    s = Shape(32, 4, 2, 8, 40)
+    ws = _stack(24, s, 2)
+    x = np.random.default_rng(25).standard_normal((6, 32))
+    full = oracle.prefix_forward(x, ws, 0, 2, KVCache(range(2), 2, 8, 16), s)
+    c = KVCache(range(2), 2, 8, 16)
+    oracle.prefix_forward(x[:5], ws, 0, 2, c, s)
+    seeded = KVCache(range(2), 2, 8, 16)
+    for l in range(2):
+        seeded.fill(l, c.k[l][:, :5].copy(), c.v[l][:, :5].copy())
+    assert seeded.length == {0: 5, 1: 5}
+    y = oracle.decode_step(x[5:6], ws, 0, 2, seeded, s)
+    np.testing.assert_allclose(y[0], full[5], rtol=1e-11, atol=1e-12)
+
+
+def test_kv_fill_closed_form_uniform_attention():
+    # W_q = W_k = 0 and every seeded key 0: the decode query at position n attends uniformly
+    # to the n seeded positions and its own. Seeded values v_j = (j + 1) * e_{(j mod d_h)} in
+    # KV head 0 and 0 in head 1; W_v = 0, so the new value is 0. With W_o = I and W_down = 0,
+    # y = x + concat(o_head0, o_head0, o_head1...) where o for query heads 0, 1 (KV head 0)
+    # is sum_j v_j / (n + 1), and 0 for query heads 2, 3 (KV head 1).
+    s = Shape(32, 4, 2, 8, 40)
+    rng = np.random.default_rng(26)
+    w = _rand_layer(rng, s)
+    w.w_q[:] = 0.0; w.w_k[:] = 0.0; w.w_v[:] = 0.0
+    w.w_o = np.eye(32); w.w_down[:] = 0.0
+    n = 11
+    kseed = np.zeros((2, n, 8))
+    vseed = np.zeros((2, n, 8))
+    for j in range(n):
+        vseed[0, j, j % 8] = j + 1.0
+    cache = KVCache([0], 2, 8, 16)
+    cache.fill(0, kseed, vseed)
+    x = rng.standard_normal((1, 32))
+    y = oracle.decode_step(x, [w], 0, 1, cache, s)
+    o0 = np.zeros(8)
+    for j in range(n):
+        o0[j % 8] += (j + 1.0) / (n + 1)
+    exp = x[0] + np.concatenate([o0, o0, np.zeros(16)])
+    np.testing.assert_allclose(y[0], exp, rtol=1e-12, atol=1e-12)
+    assert cache.length[0] == n + 1
+    np.testing.assert_array_equal(cache.v[0][:, :n], vseed)
+
+
 def test_kv_full_raises():
     s = Shape(16, 2, 1, 8, 24)
     with pytest.raises(ValueError):
