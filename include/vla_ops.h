@@ -55,7 +55,11 @@ vla_status vla_op_attention_prefill(const void* q, const void* k_plane, const vo
  * calls whose GPU work overlaps (e.g. on different streams) race on it and must be ordered
  * by the caller. The first call on a device resolves the array's device address (a
  * cudaGetSymbolAddress with that device current) and reads its SM count; make that first
- * call before any stream capture. Errors: INVALID_ARG, UNSUPPORTED, SHAPE, CUDA. */
+ * call before any stream capture. The address belongs to the device's CUDA context: after
+ * the context is destroyed and created again (cudaDeviceReset), the next call resolves it
+ * anew, so that call too should come before any capture. With 152 SMs the split count never
+ * needs to shrink for the array (splits * n_heads * (head_dim + 2) stays below 330,000
+ * floats for every supported head grouping). Errors: INVALID_ARG, UNSUPPORTED, SHAPE, CUDA. */
 vla_status vla_op_attention_decode_noalloc(const void* q, const void* k_plane, const void* v_plane, int ctx,
                                            int n_heads, int n_kv_heads, int head_dim, int max_ctx, void* out,
                                            vla_stream stream);

@@ -177,6 +177,14 @@ vla_status vla_prefix_decode_batch(vla_prefix* p, const void* hidden_in, int bat
 vla_status vla_boundary_to_host(const void* hidden_out, int n_tokens, int hidden, void* pinned_dst,
                                 vla_stream side_stream, vla_event ready, vla_event done);
 
+/* Input hand-off of a frame: copies n_tokens x hidden bf16 hidden states from page-locked
+ * host memory `pinned_src` into the device buffer `hidden_in` on `stream` (the tokens that
+ * enter block 1 of the ordered block list, Eq. 4; in the paper's pipeline they come from the
+ * vision encoder, Sec. IV-C). Asynchronous: the caller must not overwrite pinned_src before
+ * work recorded on `stream` after this call has completed. Errors: INVALID_ARG, NOT_PINNED,
+ * CUDA. */
+vla_status vla_frame_to_device(const void* pinned_src, int n_tokens, int hidden, void* hidden_in, vla_stream stream);
+
 /* Reads and clears the object's device status (blocking read; call after synchronising the
  * streams the object used). VLA_ERR_TIMEOUT if a kernel's bounded wait ran out. */
 vla_status vla_last_async_error(vla_prefix* p);

@@ -19,7 +19,7 @@ __all__ = [
     "build", "load", "VlaError", "VlaConfig", "VlaLayerWeights",
     "vla_prefix_create", "vla_prefix_destroy", "vla_kv_create", "vla_kv_destroy", "vla_kv_reset",
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
-    "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_prefix_decode_batch", "vla_boundary_to_host", "vla_last_async_error", "vla_status_str",
+    "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_prefix_decode_batch", "vla_boundary_to_host", "vla_frame_to_device", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
     "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "vla_prefix_info", "STATUS", "STAGES",
     "VlaFrameTimes", "vla_cpu_model_create", "vla_cpu_model_destroy", "vla_cpu_model_threads", "vla_cpu_model_info",
@@ -115,6 +115,7 @@ def load():
         "vla_prefix_prefill_to_host": ([P, V, I, I, I, P, V, V, V], I),
         "vla_prefix_decode_batch": ([P, V, I, I, I, ctypes.POINTER(P), V, V], I),
         "vla_boundary_to_host": ([V, I, I, V, V, V, V], I),
+        "vla_frame_to_device": ([V, I, I, V, V], I),
         "vla_last_async_error": ([P], I),
         "vla_status_str": ([I], ctypes.c_char_p),
         "vla_last_launch_count": ([P], I),
@@ -285,6 +286,11 @@ def vla_boundary_to_host(hidden_out, n_tokens: int, hidden: int, pinned_dst, sid
                          done=None):
     _check(load().vla_boundary_to_host(_ptr(hidden_out), n_tokens, hidden, _ptr(pinned_dst), _stream(side_stream),
                                        _event(ready), _event(done)), "vla_boundary_to_host")
+
+
+def vla_frame_to_device(pinned_src, n_tokens: int, hidden: int, hidden_in, stream=None):
+    _check(load().vla_frame_to_device(_ptr(pinned_src), n_tokens, hidden, _ptr(hidden_in), _stream(stream)),
+           "vla_frame_to_device")
 
 
 def vla_last_async_error(p) -> int:

@@ -1,8 +1,8 @@
 // Single-token (decode) attention on the 5th-generation tensor cores, head_dim 128.
 //
 // One thread-block cluster of `cs` CTAs per (sequence, KV head g); CTA rank r owns the contiguous key range
-// [r*ceil(ctx/cs), ...) of the context (Sec. 3.2's causal attention at one query position,
-// split over keys). Per CTA, for the G query heads of the GQA group:
+// [r*ceil(ctx/cs), ...) of the context (the attention stage of a block, Sec. IV-B, at one query
+// position, split over keys). Per CTA, for the G query heads of the GQA group:
 //   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory
 //      sized to the range (two CTAs fit on an SM, so all Hkv clusters of 16 are co-resident).
 //      Rows that predate this step are requested before griddepcontrol.wait, so the copy

@@ -185,16 +185,53 @@ cudaError_t launch_partial(dim3 grid, cudaStream_t s, const bf16* q, const bf16*
     return cudaGetLastError();
 }
 
-std::mutex g_setup_mu;
-float* g_scratch_ptr[kMaxDevices] = {};
-int g_sm_count[kMaxDevices] = {};
+typedef CUresult (*PFN_ctxGetCurrent_t)(CUcontext*);
+typedef CUresult (*PFN_ctxGetId_t)(CUcontext, unsigned long long*);
 
-// Once per device, with that device current: resolve the array's device address (host code
-// cannot use the symbol's name as a pointer) and read the SM count.
+// Unique id of the calling thread's current CUDA context (0 when there is none yet). Ids are
+// never reused within a process, so a context destroyed and created again (a device reset)
+// gets a new one.
+unsigned long long current_context_id() {
+    static PFN_ctxGetCurrent_t get_current = nullptr;
+    static PFN_ctxGetId_t get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<PFN_ctxGetCurrent_t>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<PFN_ctxGetId_t>(p);
+    });
+    if (!get_current || !get_id) return 0;
+    CUcontext c = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&c) != CUDA_SUCCESS || !c || get_id(c, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+struct DeviceSetup {
+    unsigned long long ctx_id;  // context the address below belongs to
+    float* scratch;
+    int sms;
+};
+
+std::mutex g_setup_mu;
+DeviceSetup g_setup[kMaxDevices] = {};
+
+// Once per device and context, with that device current: resolve the array's device address
+// (host code cannot use the symbol's name as a pointer) and read the SM count. The address
+// belongs to the context it was resolved in, so a new context on the device (after a device
+// reset) resolves it again.
 vla_status setup_device(int dev, float** scratch, int* sms) {
     std::lock_guard<std::mutex> lock(g_setup_mu);
-    if (!g_scratch_ptr[dev]) {
-        void* ptr = nullptr;
+    DeviceSetup& d = g_setup[dev];
+    const unsigned long long id = current_context_id();
+    if (!d.scratch || id == 0 || id != d.ctx_id) {
+        void* ptr = nullptr;  // this call also creates the device's context if there is none yet
         if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) {
             cudaGetLastError();
             return VLA_ERR_CUDA;
@@ -204,11 +241,12 @@ vla_status setup_device(int dev, float** scratch, int* sms) {
             cudaGetLastError();
             return VLA_ERR_CUDA;
         }
-        g_sm_count[dev] = n;
-        g_scratch_ptr[dev] = static_cast<float*>(ptr);
+        d.scratch = static_cast<float*>(ptr);
+        d.sms = n;
+        d.ctx_id = current_context_id();
     }
-    *scratch = g_scratch_ptr[dev];
-    *sms = g_sm_count[dev];
+    *scratch = d.scratch;
+    *sms = d.sms;
     return VLA_OK;
 }
 

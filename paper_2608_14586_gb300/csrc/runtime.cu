@@ -795,6 +795,20 @@ vla_status vla_boundary_to_host(const void* hidden_out, int n_tokens, int hidden
     return cuda_status(e);
 }
 
+vla_status vla_frame_to_device(const void* pinned_src, int n_tokens, int hidden, void* hidden_in,
+                               vla_stream stream) {
+    if (!pinned_src || !hidden_in || n_tokens < 0 || hidden <= 0) return VLA_ERR_INVALID_ARG;
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, pinned_src) != cudaSuccess) {
+        cudaGetLastError();
+        return VLA_ERR_NOT_PINNED;
+    }
+    if (attr.type != cudaMemoryTypeHost) return VLA_ERR_NOT_PINNED;
+    if (n_tokens == 0) return VLA_OK;
+    return cuda_status(cudaMemcpyAsync(hidden_in, pinned_src, (size_t)n_tokens * hidden * 2, cudaMemcpyHostToDevice,
+                                       (cudaStream_t)stream));
+}
+
 vla_status vla_last_async_error(vla_prefix* p) {
     if (!p) return VLA_ERR_INVALID_ARG;
     unsigned code = 0;

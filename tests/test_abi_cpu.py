@@ -63,6 +63,7 @@ def test_host_side_argument_errors(lib):
     assert lib.vla_prefix_prefill_to_host(None, None, 1, 0, 1, None, None, None, None) == 1
     assert lib.vla_prefix_decode_batch(None, None, 2, 0, 1, None, None, None) == 1
     assert lib.vla_boundary_to_host(None, 1, 1, None, None, None, None) == 1
+    assert lib.vla_frame_to_device(None, 1, 1, None, None) == 1
     assert lib.vla_op_gemm_bf16(None, None, 1, 1, 1, None, None) == 1
     assert lib.vla_last_async_error(None) == 1
     # unsupported shapes are refused before any allocation (head_dim 96)
@@ -84,28 +85,20 @@ def test_binding_names_match_the_header():
         assert n in vla.__all__, n
 
 
-def test_headers_are_plain_c_and_the_readme_example_compiles():
-    """Every public header compiles as C (not only C++), and the C usage example in the README
-    matches the declared signatures (wrapped in a function whose parameters supply the
-    buffers, streams and events it uses)."""
+def test_headers_are_plain_c_and_the_c_example_compiles():
+    """Every public header compiles as C (not only C++), and the C usage example
+    (tests/c_example/boundary_example.c) matches the declared signatures."""
     cc = shutil.which("gcc") or shutil.which("cc")
     if cc is None:
         pytest.skip("no C compiler")
     cuda_inc = "/usr/local/cuda/include"
     if not os.path.exists(os.path.join(cuda_inc, "cuda_runtime.h")):
         pytest.skip("CUDA headers not found")
-    with open(os.path.join(ROOT, "README.md")) as f:
-        readme = f.read()
-    m = re.search(r"```c\n(.*?)```", readme, flags=re.S)
-    assert m, "README has no C example"
-    body = "\n".join(line for line in m.group(1).splitlines() if not line.startswith("#include"))
-    src = ("#include <cuda_runtime.h>\n"
-           + "".join(f'#include "{os.path.basename(h)}"\n'
-                     for h in sorted(glob.glob(os.path.join(ROOT, "include", "*.h"))))
-           + "void example(const vla_layer_weights* layers, const void* h_in, void* h_out, void* pinned,\n"
-             "             const void* x1, void* y1, cudaStream_t stream, cudaStream_t side_stream,\n"
-             "             cudaEvent_t ready, cudaEvent_t done) {\n" + body + "\n}\n")
-    r = subprocess.run([cc, "-std=c11", "-fsyntax-only", "-Wall", "-Werror", "-x", "c", "-",
-                        "-I", os.path.join(ROOT, "include"), "-I", cuda_inc],
-                       input=src, capture_output=True, text=True)
+    for h in sorted(glob.glob(os.path.join(ROOT, "include", "*.h"))):
+        r = subprocess.run([cc, "-std=c11", "-fsyntax-only", "-Wall", "-Werror", "-x", "c", h,
+                            "-I", os.path.join(ROOT, "include"), "-I", cuda_inc], capture_output=True, text=True)
+        assert r.returncode == 0, (h, r.stderr)
+    example = os.path.join(ROOT, "tests", "c_example", "boundary_example.c")
+    r = subprocess.run([cc, "-std=c11", "-fsyntax-only", "-Wall", "-Werror", example,
+                        "-I", os.path.join(ROOT, "include"), "-I", cuda_inc], capture_output=True, text=True)
     assert r.returncode == 0, r.stderr

@@ -65,14 +65,18 @@ def test_prefill_16_blocks_2304_tokens_teacher_forced_and_partition_identity(vla
         m.close()
 
 
-def test_decode_16_blocks_context_2304_teacher_forced(vla_lib):
-    """Decode steps on the whole range (one captured graph) equal block-by-block decode bit
-    for bit; each block matches the oracle's decode step given the same input."""
+def test_decode_16_blocks_context_2304_all_64_steps(vla_lib):
+    """All 64 decode steps of the decode workload on the whole range (one captured graph)
+    equal block-by-block decode bit for bit. Against the oracle, teacher-forced (each block
+    given its GPU input) and chained (the oracle runs the 16 blocks on the step inputs). The
+    oracle takes the 64 independent step inputs of a block as one 64-token call from position
+    2304, which is the same computation as 64 single-token steps (causal mask; pinned by the
+    prefill-then-decode test of the oracle)."""
     import torch
     vla = vla_lib
     wl = synth.WORKLOADS["7b_decode16_ctx2304"]
     s, L, ctx0 = wl.shape, wl.prefix_layers, wl.prefill_ctx
-    steps, max_ctx = 3, ctx0 + 64
+    steps, max_ctx = wl.decode_steps, ctx0 + 64
     m = Model(s, L, wl.seed, max_ctx)
     try:
         kv_a = vla.vla_kv_create(m.handle, 0, L, max_ctx)
@@ -86,7 +90,7 @@ def test_decode_16_blocks_context_2304_teacher_forced(vla_lib):
             sync()
             vla.vla_kv_set_length(kv, ctx0)
         out = torch.empty((1, s.hidden), dtype=torch.bfloat16, device="cuda")
-        hs = []  # hs[t][l]: block l's input at step t (GPU, block-by-block run)
+        hs = np.empty((L + 1, steps, s.hidden))  # hs[l, t]: block l's input at step t (block by block)
         for t in range(steps):
             x = to_dev(synth.decode_hidden(t, s.hidden, wl.seed))
             vla.vla_prefix_decode(m.handle, x, 0, L, kv_a, out)
@@ -95,16 +99,32 @@ def test_decode_16_blocks_context_2304_teacher_forced(vla_lib):
                 vla.vla_prefix_decode(m.handle, h[l], l, l + 1, kv_b, h[l + 1])
             sync()
             assert torch.equal(out.view(torch.int16), h[L].view(torch.int16)), t
-            hs.append([from_dev(v) for v in h])
+            for l in range(L + 1):
+                hs[l, t] = from_dev(h[l])[0]
         assert vla.vla_last_async_error(m.handle) == 0
         assert vla.vla_kv_length(kv_a) == ctx0 + steps and vla.vla_kv_length(kv_b) == ctx0 + steps
-        cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, max_ctx)
+
+        def seeded_cache():
+            c = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, max_ctx)
+            for l in range(L):
+                c.fill(l, oracle.bf16_to_f64(ctx_bits[l][0]), oracle.bf16_to_f64(ctx_bits[l][1]))
+            return c
+
+        forced, chained = seeded_cache(), seeded_cache()
+        ref = hs[0].copy()
         for l in range(L):
-            cache.fill(l, oracle.bf16_to_f64(ctx_bits[l][0]), oracle.bf16_to_f64(ctx_bits[l][1]))
-            for t in range(steps):
-                ref = oracle.block_forward(hs[t][l], m.w64(l), cache, l, s)
-                assert rel_l2(hs[t][l + 1], ref) < REL_L2_BLOCK, (l, t)
+            tf = oracle.block_forward(hs[l], m.w64(l), forced, l, s)
+            assert rel_l2(hs[l + 1], tf) < REL_L2_BLOCK, l
+            ref = oracle.block_forward(ref, m.w64(l), chained, l, s)
+            assert rel_l2(hs[l + 1], ref) < REL_L2_BLOCK, l
             m.drop_w64()
+        for t in range(steps):
+            assert cos_sim(hs[L, t], ref[t]) > COS_FINAL, t
+        # the appended keys and values of every step, every layer
+        for l in range(L):
+            K, V = kv_planes(vla, kv_a, l, s, max_ctx)
+            assert rel_l2(from_dev(K)[:, ctx0:ctx0 + steps], chained.k[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(V)[:, ctx0:ctx0 + steps], chained.v[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
         vla.vla_kv_destroy(kv_a)
         vla.vla_kv_destroy(kv_b)
     finally:

@@ -1,0 +1,79 @@
+"""Chained parity at the full benchmark shapes: the GPU runs the range, the float64 oracle
+runs the same range on the same bits, every row and every block.
+
+* The 16-block 7B-class prefix over one 2304-token frame (6 x 320 visual + 384 text rows).
+* The 32-block 7B-class stack over one 3072-token frame (6 x 448 visual + 384 text rows),
+  cut at the split points k = 8, 16, 24 (Eq. 5-6: the boundary h^(k) of a range call must be
+  the same tensor the unpartitioned stack holds after block k).
+
+Each block's output is compared with the oracle's block output of the chain (relative L2 over
+all tokens x D), each layer's written keys and values likewise, and every boundary by cosine
+similarity. The oracle takes a few seconds per block on the host cores.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from helpers import COS_FINAL, REL_L2_BLOCK, Model, cos_sim, from_dev, kv_planes, rel_l2, sync, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_chain(vla, wl, bounds):
+    """GPU block by block (block l's output in h[l + 1]) and in range calls cut at ``bounds``;
+    the oracle chained over every block. Returns nothing; asserts as it goes."""
+    import torch
+    s, L, M = wl.shape, wl.prefix_layers, wl.n_tokens
+    m = Model(s, L, wl.seed, M)
+    try:
+        xb = synth.hidden_states(M, s.hidden, wl.seed, wl.visual_tokens, wl.visual_scale)
+        kv = vla.vla_kv_create(m.handle, 0, L, M)
+        h = [to_dev(xb)] + [torch.empty((M, s.hidden), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+        for l in range(L):
+            vla.vla_prefix_prefill(m.handle, h[l], M, l, l + 1, kv, h[l + 1])
+        # range calls [0, k1), [k1, k2), ... on a second cache: each boundary bit-equal to the
+        # block-by-block chain at the same depth
+        kv_r = vla.vla_kv_create(m.handle, 0, L, M)
+        cut = [0] + list(bounds) + [L]
+        hb = [h[0]] + [torch.empty_like(h[0]) for _ in range(len(cut) - 1)]
+        for i in range(len(cut) - 1):
+            vla.vla_prefix_prefill(m.handle, hb[i], M, cut[i], cut[i + 1], kv_r, hb[i + 1])
+        sync(300)
+        assert vla.vla_last_async_error(m.handle) == 0
+        for i in range(1, len(cut)):
+            assert torch.equal(hb[i].view(torch.int16), h[cut[i]].view(torch.int16)), cut[i]
+        vla.vla_kv_destroy(kv_r)
+
+        cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, M)
+        ref = oracle.bf16_to_f64(xb)
+        worst = 0.0
+        for l in range(L):
+            ref = oracle.block_forward(ref, m.w64(l), cache, l, s)
+            m.drop_w64()
+            got = from_dev(h[l + 1])
+            e = rel_l2(got, ref)
+            worst = max(worst, e)
+            assert e < REL_L2_BLOCK, (l, e)
+            K, V = kv_planes(vla, kv, l, s, M)
+            assert rel_l2(from_dev(K), cache.k[l]) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(V), cache.v[l]) < REL_L2_BLOCK, l
+            cache.k[l] = cache.v[l] = None  # keep host memory flat over the chain
+            if l + 1 in cut[1:]:
+                c = cos_sim(got, ref)
+                assert c > COS_FINAL, (l + 1, c)
+        vla.vla_kv_destroy(kv)
+        print(f"{wl.name}: worst per-block rel-L2 on the chain {worst:.2e}")
+    finally:
+        m.close()
+
+
+def test_prefix16_2304_tokens_chained_against_oracle(vla_lib):
+    _run_chain(vla_lib, synth.WORKLOADS["7b_prefix16_2304tok"], bounds=(8,))
+
+
+def test_stack32_3072_tokens_split_8_16_24_chained_against_oracle(vla_lib):
+    wl = synth.WORKLOADS["7b_pipeline32_3072tok"]
+    # the whole 32-block stack runs on the GPU here, cut at each split point of the sweep
+    import dataclasses
+    _run_chain(vla_lib, dataclasses.replace(wl, prefix_layers=wl.n_layers), bounds=(8, 16, 24))

@@ -72,5 +72,7 @@ def test_reference_arm_prints_on_rank_zero_only():
     assert line["impl"] == "reference" and line["n_gpus"] == 2
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
-    # 512 sampled tokens of one block in 0.5 s, extrapolated to the 16-block prefix
-    assert abs(line["value"] - 512 / (0.5 * 16)) < 1e-9
+    # one block over the whole 2304-token frame in 0.5 s per step, taken x16 for the 16-block
+    # prefix; the reported step time is the measured sample step
+    assert abs(line["value"] - 2304 / (0.5 * 16)) < 1e-9
+    assert abs(line["ms_per_step"] - 500.0) < 1e-9
