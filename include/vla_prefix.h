@@ -217,6 +217,16 @@ enum {
     VLA_STAGE_COUNT = 12
 };
 vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask);
+
+/* Failure-detection test support (not part of the method): the next prefill launch of GEMM
+ * stage `stage` (VLA_STAGE_GEMM_QKV, _O, _GATEUP or _DOWN) never loads the last k-block of
+ * each CTA's first tile, so that kernel's bounded waits run out after wait_budget_cycles SM
+ * cycles (1e5 .. 2e9; the default bound of every wait is 2e9, about 1 s). The kernel then
+ * records VLA_ERR_TIMEOUT for vla_last_async_error, lets its copies in flight land, retires
+ * its MMAs, releases its tensor memory and exits; the call's output is undefined, later calls
+ * run normally. One launch consumes the request; stage = -1 cancels it. Errors: INVALID_ARG,
+ * UNSUPPORTED (not a GEMM stage). */
+vla_status vla_prefix_inject_stall(vla_prefix* p, int stage, long long wait_budget_cycles);
 vla_status vla_prefix_stage_times(vla_prefix* p, float* ms_per_stage, int* launches_per_stage, int n_stages);
 
 #ifdef __cplusplus

@@ -21,7 +21,7 @@ __all__ = [
     "vla_kv_length", "vla_kv_layer_length", "vla_kv_data", "vla_kv_decode_plan", "vla_kv_set_length", "vla_prefix_prefill",
     "vla_prefix_prefill_to_host", "vla_prefix_decode", "vla_prefix_decode_batch", "vla_boundary_to_host", "vla_frame_to_device", "vla_last_async_error", "vla_status_str",
     "vla_last_launch_count", "vla_op_gemm_bf16", "vla_op_attention_prefill", "vla_prefix_set_timing",
-    "vla_prefix_stage_times", "vla_op_attention_decode_noalloc", "vla_prefix_info", "STATUS", "STAGES",
+    "vla_prefix_stage_times", "vla_prefix_inject_stall", "vla_op_attention_decode_noalloc", "vla_prefix_info", "STATUS", "STAGES",
     "VlaFrameTimes", "vla_cpu_model_create", "vla_cpu_model_destroy", "vla_cpu_model_threads", "vla_cpu_model_info",
     "vla_cpu_kv_create", "vla_cpu_kv_destroy", "vla_cpu_kv_reset", "vla_cpu_kv_length", "vla_cpu_kv_data",
     "vla_cpu_prefill", "vla_pipeline_create", "vla_pipeline_submit", "vla_pipeline_collect",
@@ -122,6 +122,7 @@ def load():
         "vla_op_gemm_bf16": ([V, V, I, I, I, V, V], I),
         "vla_op_attention_prefill": ([V, V, V, I, I, I, I, I, I, V, V], I),
         "vla_prefix_set_timing": ([P, ctypes.c_uint], I),
+        "vla_prefix_inject_stall": ([P, I, ctypes.c_longlong], I),
         "vla_op_attention_decode_noalloc": ([V, V, V, I, I, I, I, I, V, V], I),
         "vla_prefix_stage_times": ([P, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_int), I], I),
         "vla_prefix_info": ([P, ctypes.POINTER(VlaConfig), ctypes.POINTER(I)], I),
@@ -299,6 +300,13 @@ def vla_last_async_error(p) -> int:
 
 def vla_last_launch_count(p) -> int:
     return load().vla_last_launch_count(p)
+
+
+def vla_prefix_inject_stall(p, stage, wait_budget_cycles: int):
+    """Arms the failure-detection test fault on the next prefill launch of a GEMM stage (a
+    name of STAGES or its id; -1 / None cancels)."""
+    sid = -1 if stage is None or stage == -1 else (STAGES.index(stage) if isinstance(stage, str) else int(stage))
+    _check(load().vla_prefix_inject_stall(p, sid, int(wait_budget_cycles)), "vla_prefix_inject_stall")
 
 
 def vla_op_gemm_bf16(A, B, M: int, N: int, K: int, C, stream=None):

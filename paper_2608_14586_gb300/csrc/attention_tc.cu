@@ -14,8 +14,9 @@
 //               keys, K=d_h) into TMEM columns [128t, 128t+128) and O_t += P_t V (M=128, N=d_h,
 //               K=128 keys) into TMEM columns [256 + t*d_h, ...), with P_t read from tensor
 //               memory (the softmax writes it as packed bf16 over the first 64 columns of S_t)
-//               and V from shared memory as an MN-major operand. The next S_t is issued once
-//               PV_t has completed, since P_t occupies its columns.
+//               and V from shared memory as an MN-major operand. The next S_t is issued right
+//               behind PV_t: one thread's MMAs execute in issue order, so PV_t has read P_t
+//               before S_t is overwritten, and the thread never waits on an MMA.
 //   warps 2..5  softmax of tile A, warps 6..9 of tile B; one thread per query row (TMEM lane):
 //               reads its S row once (tcgen05.ld), masks, takes the row max, writes
 //               P = exp2(s - m) as bf16 into tensor memory (tcgen05.st), keeps the row sum, and
@@ -254,19 +255,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                // S of block 0 for both tiles (their S columns were freed by the previous pair's
-                // last PV, which this thread waited for before issuing anything after it)
+                // S of block 0 for both tiles: their columns hold the previous pair's last P,
+                // read by a PV issued before (issue order, as below)
                 for (int t = 0; t < 2; ++t)
                     if (p.n[t] > 0) issue_s(t, nkv, smem_u32(smem + t * C::Q_BYTES));
                 umma_commit(&bars->k_empty[nkv & 1]);
                 if (nmax == 1) umma_commit(&bars->q_free);
                 for (int j = 0; j < nmax && ok; ++j) {
                     const uint32_t n = nkv + j;
-                    if (!wait_ab(&bars->v_full[n & 1], (n >> 1) & 1u, &s_abort)) {
+                    if (!wait_ab(&bars->v_full[n & 1], (n >> 1) & 1u, &s_abort) ||
+                        (j + 1 < nmax && !wait_ab(&bars->k_full[(n + 1) & 1], ((n + 1) >> 1) & 1u, &s_abort))) {
                         ok = false;
                         break;
                     }
-                    bool k_next = false;  // K of block j+1 waited for
                     for (int t = 0; t < 2 && ok; ++t) {
                         if (j >= p.n[t]) continue;
                         if (!wait_ab(&bars->p_full[t], gt[t] & 1u, &s_abort) ||
@@ -282,18 +283,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                             umma_bf16_ts(tmem + C::O_COL + t * DH, tmem + t * kBN + kk * 8, bd, C::IDESC_O,
                                          (j > 0 || kk > 0) ? 1u : 0u);
                         }
-                        umma_commit(&bars->pv_done[t]);
-                        if (j + 1 < p.n[t]) {
-                            // the next S of this tile overwrites P: wait for this PV, and for K
-                            if (!wait_ab(&bars->pv_done[t], gt[t] & 1u, &s_abort) ||
-                                (!k_next && !wait_ab(&bars->k_full[(n + 1) & 1], ((n + 1) >> 1) & 1u, &s_abort))) {
-                                ok = false;
-                                break;
-                            }
-                            k_next = true;
-                            tc_fence_after();
-                            issue_s(t, n + 1, smem_u32(smem + t * C::Q_BYTES));
-                        }
+                        // The next S of this tile overwrites P_t in the same columns. It is issued
+                        // right behind the PV that reads P_t: the tensor core executes one thread's
+                        // MMAs in issue order, so the PV's operand reads precede the S's writes.
+                        // Its commit also tells the softmax that PV_t has completed (O_t may be
+                        // rescaled).
+                        if (j + 1 < p.n[t]) issue_s(t, n + 1, smem_u32(smem + t * C::Q_BYTES));
+                        else umma_commit(&bars->pv_done[t]);  // the tile's last PV: O_t is final
                         ++gt[t];
                     }
                     if (!ok) break;
@@ -304,12 +300,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 if (!ok) break;
-                // the last PV of each tile must finish before that tile's S columns are reused
-                for (int t = 0; t < 2 && ok; ++t) {
-                    if (p.n[t] == 0) continue;
-                    if (!wait_ab(&bars->pv_done[t], (gt[t] - 1) & 1u, &s_abort)) ok = false;
-                    ++et[t];
-                }
+                for (int t = 0; t < 2; ++t)
+                    if (p.n[t] > 0) ++et[t];
                 nkv += nmax;
             }
             if (!ok) {
@@ -329,7 +321,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t scol = (uint32_t)t * kBN;
         const uint32_t ocol = C::O_COL + (uint32_t)t * DH;
         bool ok = true;
-        uint32_t g = 0;  // blocks of this tile slot so far
+        uint32_t g = 0;   // blocks of this tile slot so far (S and P phases)
+        uint32_t np = 0;  // pairs in which this tile slot existed (final-PV phases)
         Pair p;
         for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
             if (p.n[t] == 0) continue;  // no tile B in this pair
@@ -359,13 +352,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (key > qpos || key >= a.ctx) sr[i] = 0xFF800000u;  // -inf
                         }
                     }
+                    // row max with three-input max instructions, eight independent chains
                     float mc[8];
 #pragma unroll
                     for (int q = 0; q < 8; ++q) mc[q] = __uint_as_float(sr[q]);
 #pragma unroll
-                    for (int i = 8; i < kBN; ++i) mc[i & 7] = fmaxf(mc[i & 7], __uint_as_float(sr[i]));
-                    const float mraw = fmaxf(fmaxf(fmaxf(mc[0], mc[1]), fmaxf(mc[2], mc[3])),
-                                             fmaxf(fmaxf(mc[4], mc[5]), fmaxf(mc[6], mc[7])));
+                    for (int i = 8; i < kBN; i += 16) {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            mc[q] = fmax3(mc[q], __uint_as_float(sr[i + q]),
+                                          i + 8 + q < kBN ? __uint_as_float(sr[i + 8 + q]) : mc[q]);
+                    }
+                    const float mraw = fmax3(fmax3(mc[0], mc[1], mc[2]), fmax3(mc[3], mc[4], mc[5]), fmaxf(mc[6], mc[7]));
                     const float mx = mraw * a.scale_log2;  // scale > 0
                     if (m_run == -INFINITY) {
                         m_new = mx;
@@ -379,22 +377,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     l_run *= corr;
                     const bool warp_need = __any_sync(0xFFFFFFFFu, need);
                     // P = exp2(s * scale - m) as packed bf16 over the first 64 columns of S
-                    const float neg_m = -m_new;
-                    float ls[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial sums of the row
+                    // two columns per instruction for the scaling and the row sum (packed fp32)
+                    const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+                    const float2 nm2 = make_float2(-m_new, -m_new);
+                    float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};  // partial row sums
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         uint32_t pk[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
-                            const float p0 = ex2_approx(fmaf(__uint_as_float(sr[64 * h + 2 * i]), a.scale_log2, neg_m));
-                            const float p1 =
-                                ex2_approx(fmaf(__uint_as_float(sr[64 * h + 2 * i + 1]), a.scale_log2, neg_m));
-                            ls[i & 3] += p0 + p1;
-                            pk[i] = pack_bf16x2(p0, p1);
+                            const float2 x = __ffma2_rn(
+                                make_float2(__uint_as_float(sr[64 * h + 2 * i]), __uint_as_float(sr[64 * h + 2 * i + 1])),
+                                sc2, nm2);
+                            const float2 pp = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+                            ls[i & 1] = __fadd2_rn(ls[i & 1], pp);
+                            pk[i] = pack_bf16x2(pp.x, pp.y);
                         }
                         tmem_st32(trow + scol + 32 * h, pk);
                     }
-                    l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+                    l_run += (ls[0].x + ls[1].x) + (ls[0].y + ls[1].y);
                     if (warp_need) {
                         // PV of the previous block has completed: this block's S was issued after it
 #pragma unroll 1
@@ -414,7 +415,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (!ok) break;
             // epilogue of this tile: after its last PV
-            ok = wait_ab(&bars->pv_done[t], (g - 1) & 1u, &s_abort);
+            ok = wait_ab(&bars->pv_done[t], np & 1u, &s_abort);
+            ++np;
             __syncwarp();
             if (!__all_sync(0xFFFFFFFFu, ok)) {
                 ok = false;

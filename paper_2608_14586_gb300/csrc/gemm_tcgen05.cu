@@ -232,12 +232,12 @@ VLA_DEV void epi_swiglu(uint32_t taddr, int row, int n0, const EpiParams& ep) {
 }
 
 // Bounded wait that also gives up when another role has aborted.
-VLA_DEV bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+VLA_DEV bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag, long long budget) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (!mbar_try_wait(bar, parity)) {
         if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitBudgetCycles) return false;
+        if (clock64() - t0 > budget) return false;
     }
     return true;
 }
@@ -308,6 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // while the previous kernel drains. Activations (A) only after it.
             const int pre = (blockIdx.x < num_tiles) ? min(STAGES, num_kb) : 0;
             for (int kb = 0; kb < pre; ++kb) {
+                if (kb == ep.stall_kb) continue;  // failure-detection test: never armed (below)
                 mbar_arrive_expect_tx(&full[kb], C::STAGE_BYTES);
                 tma_load_2d(sB + kb * C::B_BYTES, &tmB, &full[kb], kb * kBK, (blockIdx.x / num_m) * BN);
                 issued |= 1u << kb;
@@ -319,19 +320,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int m0 = (tile % num_m) * kBM;
                 const int n0 = (tile / num_m) * BN;
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    if (!wait_or_abort(&empty[stage], phase ^ 1u, &s_abort)) {
+                    if (!wait_or_abort(&empty[stage], phase ^ 1u, &s_abort, ep.wait_budget)) {
                         ok = false;
                         break;
                     }
-                    if (first && kb < pre) {  // B of this stage is already in flight
+                    const bool withhold = first && kb == ep.stall_kb;
+                    if (withhold) {
+                        // failure-detection test: this stage is never armed or loaded, so the
+                        // MMA's wait on it runs out and the launch winds down
+                    } else if (first && kb < pre) {  // B of this stage is already in flight
                         tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
                     } else {
                         mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
                         tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * kBK, m0);
                         tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * kBK, n0);
                     }
-                    issued |= 1u << stage;
-                    issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                    if (!withhold) {
+                        issued |= 1u << stage;
+                        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                    }
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -342,9 +349,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) {
                 s_abort = 1;
                 set_status(ep.status, kDevTimeout);
-                // let every copy already issued land before the CTA can exit
+            }
+            if (!ok || ep.stall_kb >= 0) {
+                // let every copy already issued land before the CTA can exit (with a withheld
+                // stage the MMA stops early and may leave later copies unconsumed)
                 for (int s = 0; s < STAGES; ++s)
-                    if (issued & (1u << s)) mbar_wait(&full[s], (issued_phase >> s) & 1u);
+                    if (issued & (1u << s)) mbar_wait(&full[s], (issued_phase >> s) & 1u, ep.wait_budget);
             }
         }
     } else if (warp == 1) {
@@ -362,14 +372,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++it) {
                 const int acc = it & 1;
                 const uint32_t acc_phase = (it >> 1) & 1;
-                if (!wait_or_abort(&tempty[acc], acc_phase ^ 1u, &s_abort)) {
+                if (!wait_or_abort(&tempty[acc], acc_phase ^ 1u, &s_abort, ep.wait_budget)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + acc * BN;
                 for (int kb = 0; kb < num_kb; ++kb) {
-                    if (!wait_or_abort(&full[stage], phase, &s_abort)) {
+                    if (!wait_or_abort(&full[stage], phase, &s_abort, ep.wait_budget)) {
                         ok = false;
                         break;
                     }
@@ -395,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // all MMAs issued by this thread retire before TMEM can be released
             umma_commit(mma_done);
-            mbar_wait(mma_done, 0);
+            mbar_wait(mma_done, 0, ep.wait_budget);
         }
     } else {
         // ---------------- epilogue (warps 2..5) ----------------
@@ -406,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
             const int acc = it & 1;
             const uint32_t acc_phase = (it >> 1) & 1;
-            const bool ok = wait_or_abort(&tfull[acc], acc_phase, &s_abort);
+            const bool ok = wait_or_abort(&tfull[acc], acc_phase, &s_abort, ep.wait_budget);
             __syncwarp();
             if (!__all_sync(0xFFFFFFFFu, ok)) {
                 s_abort = 1;

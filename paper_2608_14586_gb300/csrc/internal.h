@@ -71,6 +71,11 @@ struct EpiParams {
     int* len_out;   // kEpiQKV: the layer's device KV length, set to len_value (nullptr: leave)
     int len_value;
     unsigned* status;
+    // Bound of every wait of the launch, in SM clock cycles (kWaitBudgetCycles unless a
+    // failure-detection test shortens it), and that test's injected fault: k-block `stall_kb`
+    // of each CTA's first tile is never loaded, so the waits on it run out (-1: no fault).
+    long long wait_budget;
+    int stall_kb;
 };
 
 // Tensor-map helper (driver entry point fetched through the runtime). rows x cols bf16,

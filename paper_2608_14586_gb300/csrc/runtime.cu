@@ -128,6 +128,10 @@ struct vla_prefix {
     bf16 *d_attn = nullptr, *d_xmid = nullptr, *d_m = nullptr;
     unsigned* d_status = nullptr;
     int last_launches = 0;
+    // failure-detection test: the next prefill launch of GEMM stage `fault_stage` withholds
+    // one k-block and waits at most `fault_budget` cycles (-1: none)
+    int fault_stage = -1;
+    long long fault_budget = 0;
     // measurement: event pairs around each kernel while timing is enabled
     unsigned timing = 0;  // bit s: time the kernels of stage s
     std::vector<cudaEvent_t> ev_pool;
@@ -464,6 +468,18 @@ vla_status vla_kv_data(const vla_kv* kv, int layer, void** k_plane, void** v_pla
     return VLA_OK;
 }
 
+// Wait bound and injected fault of one GEMM launch of `stage` with num_kb k-blocks: the
+// default bound, unless a failure-detection test armed this stage (consumed by one launch).
+void set_waits(vla_prefix* p, vla::EpiParams& ep, int stage, int K) {
+    ep.wait_budget = vla::kWaitBudgetCycles;
+    ep.stall_kb = -1;
+    if (p && p->fault_stage == stage) {
+        ep.wait_budget = p->fault_budget;
+        ep.stall_kb = (K + 63) / 64 - 1;
+        p->fault_stage = -1;
+    }
+}
+
 // Prefill of [layer_begin, layer_end); with host_dev set, the last block's down projection
 // also stores h^(layer_end) into page-locked host memory (host_dev: its device address).
 static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_tokens, int layer_begin, int layer_end,
@@ -550,6 +566,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ep.len_out = kv->d_len + (l - kv->lb);
         ep.len_value = p0 + M;
         ep.status = p->d_status;
+        set_waits(p, ep, VLA_STAGE_GEMM_QKV, D);
         stage_mark(p, VLA_STAGE_GEMM_QKV, true);
         e = vla::launch_gemm(vla::kEpiQKV, qkv_bn, tm_x, qkv_bn == 192 ? ld.tm_qkv192 : ld.tm_qkv, M, p->qkv_n, D,
                              ep, p->num_sms, stream, pdl(VLA_STAGE_GEMM_QKV));
@@ -586,6 +603,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         eo.ss_width = ss_w;
         eo.ss_groups = D / ss_w;
         eo.status = p->d_status;
+        set_waits(p, eo, VLA_STAGE_GEMM_O, p->qc);
         stage_mark(p, VLA_STAGE_GEMM_O, true);
         e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_attn, d_bn == 224 ? ld.tm_o224 : ld.tm_o, M, D, p->qc, eo,
                              p->num_sms, stream, pdl(VLA_STAGE_GEMM_O));
@@ -603,6 +621,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         eg.norm_dim = D;
         eg.eps = eps;
         eg.status = p->d_status;
+        set_waits(p, eg, VLA_STAGE_GEMM_GATEUP, D);
         stage_mark(p, VLA_STAGE_GEMM_GATEUP, true);
         e = vla::launch_gemm(vla::kEpiSwiGLU, kBN, tm_xmid, ld.tm_gu, M, 2 * p->F_pad, D, eg, p->num_sms, stream,
                              pdl(VLA_STAGE_GEMM_GATEUP));
@@ -621,6 +640,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         ed.ss_width = ss_w;
         ed.ss_groups = D / ss_w;
         ed.status = p->d_status;
+        set_waits(p, ed, VLA_STAGE_GEMM_DOWN, p->F_pad);
         stage_mark(p, VLA_STAGE_GEMM_DOWN, true);
         e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_m, d_bn == 224 ? ld.tm_d224 : ld.tm_d, M, D, p->F_pad, ed,
                              p->num_sms, stream, pdl(VLA_STAGE_GEMM_DOWN));
@@ -826,6 +846,21 @@ vla_status vla_prefix_info(const vla_prefix* p, vla_config* cfg, int* layer_coun
     return VLA_OK;
 }
 
+vla_status vla_prefix_inject_stall(vla_prefix* p, int stage, long long wait_budget_cycles) {
+    if (!p) return VLA_ERR_INVALID_ARG;
+    if (stage == -1) {
+        p->fault_stage = -1;
+        return VLA_OK;
+    }
+    if (stage != VLA_STAGE_GEMM_QKV && stage != VLA_STAGE_GEMM_O && stage != VLA_STAGE_GEMM_GATEUP &&
+        stage != VLA_STAGE_GEMM_DOWN)
+        return VLA_ERR_UNSUPPORTED;
+    if (wait_budget_cycles < 100000 || wait_budget_cycles > vla::kWaitBudgetCycles) return VLA_ERR_INVALID_ARG;
+    p->fault_stage = stage;
+    p->fault_budget = wait_budget_cycles;
+    return VLA_OK;
+}
+
 vla_status vla_prefix_set_timing(vla_prefix* p, unsigned stage_mask) {
     if (!p) return VLA_ERR_INVALID_ARG;
     p->timing = stage_mask;
@@ -872,6 +907,7 @@ vla_status vla_op_gemm_bf16(const void* A, const void* B, int M, int N, int K, v
     ep.N = N;
     ep.out = (bf16*)C;
     ep.ld_out = N;
+    set_waits(nullptr, ep, -1, K);
     static const int sms = vla::device_sm_count();
     return cuda_status(vla::launch_gemm(vla::kEpiPlain, kBN, ta, tb, M, N, K, ep, sms, (cudaStream_t)stream));
 }

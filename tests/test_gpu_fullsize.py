@@ -110,21 +110,22 @@ def test_decode_16_blocks_context_2304_all_64_steps(vla_lib):
                 c.fill(l, oracle.bf16_to_f64(ctx_bits[l][0]), oracle.bf16_to_f64(ctx_bits[l][1]))
             return c
 
+        # teacher-forced (each block on its GPU input): the per-block bar, outputs and the keys
+        # and values each step appended; chained (the oracle's own run of the 16 blocks): every
+        # step's hidden state after every block within the final-cosine bar (bf16 hidden states
+        # between blocks make the chain drift by ~1e-3 per block, see test_gpu_parity_chained)
         forced, chained = seeded_cache(), seeded_cache()
         ref = hs[0].copy()
         for l in range(L):
             tf = oracle.block_forward(hs[l], m.w64(l), forced, l, s)
             assert rel_l2(hs[l + 1], tf) < REL_L2_BLOCK, l
-            ref = oracle.block_forward(ref, m.w64(l), chained, l, s)
-            assert rel_l2(hs[l + 1], ref) < REL_L2_BLOCK, l
-            m.drop_w64()
-        for t in range(steps):
-            assert cos_sim(hs[L, t], ref[t]) > COS_FINAL, t
-        # the appended keys and values of every step, every layer
-        for l in range(L):
             K, V = kv_planes(vla, kv_a, l, s, max_ctx)
-            assert rel_l2(from_dev(K)[:, ctx0:ctx0 + steps], chained.k[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
-            assert rel_l2(from_dev(V)[:, ctx0:ctx0 + steps], chained.v[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(K)[:, ctx0:ctx0 + steps], forced.k[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(V)[:, ctx0:ctx0 + steps], forced.v[l][:, ctx0:ctx0 + steps]) < REL_L2_BLOCK, l
+            ref = oracle.block_forward(ref, m.w64(l), chained, l, s)
+            m.drop_w64()
+            for t in range(steps):
+                assert cos_sim(hs[l + 1, t], ref[t]) > COS_FINAL, (l, t)
         vla.vla_kv_destroy(kv_a)
         vla.vla_kv_destroy(kv_b)
     finally:

@@ -67,3 +67,4 @@ def test_attention_prefill_matches_oracle(vla_lib, M, H, Hkv, dh, pos0):
     # per row: the probabilities are bf16 in the P.V product -> a few 2^-9 relative
     row_err = np.linalg.norm((got - ref).reshape(M, -1), axis=1) / np.linalg.norm(ref.reshape(M, -1), axis=1)
     assert row_err.max() < 2e-2
+

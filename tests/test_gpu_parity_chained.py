@@ -6,9 +6,16 @@ runs the same range on the same bits, every row and every block.
   cut at the split points k = 8, 16, 24 (Eq. 5-6: the boundary h^(k) of a range call must be
   the same tensor the unpartitioned stack holds after block k).
 
-Each block's output is compared with the oracle's block output of the chain (relative L2 over
-all tokens x D), each layer's written keys and values likewise, and every boundary by cosine
-similarity. The oracle takes a few seconds per block on the host cores.
+Two comparisons per block. Teacher-forced: the oracle runs the block on the GPU's own input
+to it (exact bf16 values) at sampled query rows, with every row's key and value (all of which
+attention needs), and the block's output at those rows and its whole written K/V planes must be
+within the per-block relative L2 bar: this is the error one block adds. Chained: the oracle runs
+the whole range on the frame, and the GPU's hidden state after every block (each a possible
+split point k) must have cosine similarity >= 0.999 with it. The chain's relative L2 is printed,
+not bounded per block: with bf16 hidden states between blocks (Eq. 11's b = 2) every block adds
+its rounding to the residual stream, so the chain's distance from the float64 result grows
+with depth (about 1e-3 per block at these shapes) while each block stays within its own bar.
+The full oracle takes a few seconds per block on the host cores.
 """
 import numpy as np
 import pytest
@@ -20,9 +27,11 @@ from helpers import COS_FINAL, REL_L2_BLOCK, Model, cos_sim, from_dev, kv_planes
 pytestmark = pytest.mark.gpu
 
 
-def _run_chain(vla, wl, bounds):
+def _run_chain(vla, wl, bounds, cos_depth):
     """GPU block by block (block l's output in h[l + 1]) and in range calls cut at ``bounds``;
-    the oracle chained over every block. Returns nothing; asserts as it goes."""
+    the oracle chained over every block. The chain's cosine bar holds at every depth up to
+    ``cos_depth`` (the deepest boundary the workload hands off); deeper blocks are run and
+    reported. Returns nothing; asserts as it goes."""
     import torch
     s, L, M = wl.shape, wl.prefix_layers, wl.n_tokens
     m = Model(s, L, wl.seed, M)
@@ -45,35 +54,41 @@ def _run_chain(vla, wl, bounds):
             assert torch.equal(hb[i].view(torch.int16), h[cut[i]].view(torch.int16)), cut[i]
         vla.vla_kv_destroy(kv_r)
 
+        rows = sorted(set([0, 1, M - 2, M - 1, wl.visual_tokens - 1, wl.visual_tokens] +
+                          np.random.default_rng(5).choice(M, 24, replace=False).tolist()))
         cache = oracle.KVCache(range(L), s.n_kv_heads, s.head_dim, M)
         ref = oracle.bf16_to_f64(xb)
-        worst = 0.0
+        chain = []
         for l in range(L):
-            ref = oracle.block_forward(ref, m.w64(l), cache, l, s)
-            m.drop_w64()
+            w = m.w64(l)
             got = from_dev(h[l + 1])
-            e = rel_l2(got, ref)
-            worst = max(worst, e)
-            assert e < REL_L2_BLOCK, (l, e)
+            # teacher-forced: the block on the GPU's input, sampled rows and the whole K/V planes
+            y_tf, k_tf, v_tf = oracle.block_forward_rows(from_dev(h[l]), w, s, rows)
+            assert rel_l2(got[rows], y_tf) < REL_L2_BLOCK, l
             K, V = kv_planes(vla, kv, l, s, M)
-            assert rel_l2(from_dev(K), cache.k[l]) < REL_L2_BLOCK, l
-            assert rel_l2(from_dev(V), cache.v[l]) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(K), k_tf) < REL_L2_BLOCK, l
+            assert rel_l2(from_dev(V), v_tf) < REL_L2_BLOCK, l
+            # chained: the oracle's own run of blocks [0, l]
+            ref = oracle.block_forward(ref, w, cache, l, s)
             cache.k[l] = cache.v[l] = None  # keep host memory flat over the chain
-            if l + 1 in cut[1:]:
-                c = cos_sim(got, ref)
+            m.drop_w64()
+            c = cos_sim(got, ref)
+            chain.append(rel_l2(got, ref))
+            if l + 1 <= cos_depth:
                 assert c > COS_FINAL, (l + 1, c)
         vla.vla_kv_destroy(kv)
-        print(f"{wl.name}: worst per-block rel-L2 on the chain {worst:.2e}")
+        print(f"{wl.name}: rel-L2 of the chain after each block: " + " ".join(f"{e:.1e}" for e in chain))
     finally:
         m.close()
 
 
 def test_prefix16_2304_tokens_chained_against_oracle(vla_lib):
-    _run_chain(vla_lib, synth.WORKLOADS["7b_prefix16_2304tok"], bounds=(8,))
+    _run_chain(vla_lib, synth.WORKLOADS["7b_prefix16_2304tok"], bounds=(8,), cos_depth=16)
 
 
 def test_stack32_3072_tokens_split_8_16_24_chained_against_oracle(vla_lib):
     wl = synth.WORKLOADS["7b_pipeline32_3072tok"]
-    # the whole 32-block stack runs on the GPU here, cut at each split point of the sweep
+    # the whole 32-block stack runs on the GPU here, cut at each split point of the sweep; the
+    # prefix handed off is [0, k) with k <= 24
     import dataclasses
-    _run_chain(vla_lib, dataclasses.replace(wl, prefix_layers=wl.n_layers), bounds=(8, 16, 24))
+    _run_chain(vla_lib, dataclasses.replace(wl, prefix_layers=wl.n_layers), bounds=(8, 16, 24), cos_depth=24)
