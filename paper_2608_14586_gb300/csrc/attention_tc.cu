@@ -6,8 +6,8 @@
 // each a PAIR of query tiles of one head (tile A = 128 query rows, tile B = the next 128),
 // numbered longest first and dealt to the CTAs in a snake so every CTA gets a similar number
 // of key blocks. Both tiles read the same key/value blocks, which are loaded once for the pair.
-//   warp 0      TMA: the pair's two Q tiles, then K and V blocks of 128 keys through two 2-stage
-//               rings shared by the two tiles. K/V come from the layer's cache through a 3-D
+//   warp 0      TMA: the pair's two Q tiles, then K and V blocks of 128 keys through a 2-stage K
+//               ring and a 3-stage V ring shared by the two tiles. K/V come from the layer's cache through a 3-D
 //               tensor map whose key extent ends at the context length, so keys past it arrive
 //               as zeros.
 //   warp 1      TMEM allocation; one thread issues, per tile t, S_t = Q_t K^T (M=128, N=128
@@ -45,7 +45,7 @@ struct AttnCfg {
     static constexpr uint32_t Q_BYTES = KCH * CHUNK;
     static constexpr uint32_t KV_BYTES = KCH * CHUNK;
     static constexpr int K_STAGES = 2;
-    static constexpr int V_STAGES = 2;
+    static constexpr int V_STAGES = 3;
     static constexpr uint32_t OFF_K = 2 * Q_BYTES;  // Q of tile A, then of tile B
     static constexpr uint32_t OFF_V = OFF_K + K_STAGES * KV_BYTES;
     static constexpr uint32_t OFF_BAR = OFF_V + V_STAGES * KV_BYTES;
@@ -57,7 +57,7 @@ struct AttnCfg {
 };
 
 struct Bars {
-    uint64_t q_full, q_free, k_full[2], k_empty[2], v_full[2], v_empty[2];
+    uint64_t q_full, q_free, k_full[2], k_empty[2], v_full[3], v_empty[3];
     uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];  // per tile
     uint64_t mma_done;
     uint32_t tmem_slot;
@@ -121,9 +121,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         mbar_init(&bars->q_full, 1);
         mbar_init(&bars->q_free, 1);
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < 3; ++b) {
             mbar_init(&bars->v_full[b], 1);
             mbar_init(&bars->v_empty[b], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->k_full[b], 1);
             mbar_init(&bars->k_empty[b], 1);
             mbar_init(&bars->s_full[b], 1);
@@ -196,8 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                     if (jv < nmax) {  // V runs ahead of K as far as its ring allows
-                        const int b = nv & 1;
-                        const uint32_t n = nv >> 1;
+                        const int b = (int)(nv % 3u);
+                        const uint32_t n = nv / 3u;
                         if (mbar_try_wait(&bars->v_empty[b], (n & 1u) ^ 1u)) {
                             mbar_arrive_expect_tx(&bars->v_full[b], C::KV_BYTES);
                             for (int c = 0; c < C::KCH; ++c)
@@ -224,8 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // every copy this thread issued lands before the CTA can exit
             if (issued_q) mbar_wait(&bars->q_full, ph_q);
-            for (int b = 0; b < 2; ++b) {
-                if (issued_k & (1u << b)) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
+            for (int b = 0; b < 3; ++b) {
+                if (b < 2 && (issued_k & (1u << b))) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
                 if (issued_v & (1u << b)) mbar_wait(&bars->v_full[b], (ph_v >> b) & 1u);
             }
         }
@@ -263,7 +265,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (nmax == 1) umma_commit(&bars->q_free);
                 for (int j = 0; j < nmax && ok; ++j) {
                     const uint32_t n = nkv + j;
-                    if (!wait_ab(&bars->v_full[n & 1], (n >> 1) & 1u, &s_abort) ||
+                    const uint32_t vs = n % 3u;  // V ring slot of block n, phase (n / 3) & 1
+                    if (!wait_ab(&bars->v_full[vs], (n / 3u) & 1u, &s_abort) ||
                         (j + 1 < nmax && !wait_ab(&bars->k_full[(n + 1) & 1], ((n + 1) >> 1) & 1u, &s_abort))) {
                         ok = false;
                         break;
@@ -276,13 +279,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t sV = smem_u32(smem + C::OFF_V + (n & 1) * C::KV_BYTES);
+                        const uint32_t sV = smem_u32(smem + C::OFF_V + vs * C::KV_BYTES);
 #pragma unroll
                         for (int kk = 0; kk < kBN / 16; ++kk) {
                             const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
                             umma_bf16_ts(tmem + C::O_COL + t * DH, tmem + t * kBN + kk * 8, bd, C::IDESC_O,
                                          (j > 0 || kk > 0) ? 1u : 0u);
                         }
+                        // the block's last PV: V_j's slot is free once it completes (committed
+                        // before the next S, so the producer can refill it while that S runs)
+                        if (t == 1 || j >= p.n[1]) umma_commit(&bars->v_empty[vs]);
                         // The next S of this tile overwrites P_t in the same columns. It is issued
                         // right behind the PV that reads P_t: the tensor core executes one thread's
                         // MMAs in issue order, so the PV's operand reads precede the S's writes.
@@ -293,7 +299,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ++gt[t];
                     }
                     if (!ok) break;
-                    umma_commit(&bars->v_empty[n & 1]);
                     if (j + 1 < nmax) {
                         umma_commit(&bars->k_empty[(n + 1) & 1]);
                         if (j + 2 == nmax) umma_commit(&bars->q_free);  // the pair's last S was just issued
@@ -381,20 +386,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
                     const float2 nm2 = make_float2(-m_new, -m_new);
                     float2 ls[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};  // partial row sums
+                    // packed P in four 16-column stores, waited on once: the packed words take
+                    // the place of the S values they replace, so fewer registers are live
+                    uint32_t pk[64];
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        uint32_t pk[32];
+                    for (int h = 0; h < 4; ++h) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float2 x = __ffma2_rn(
-                                make_float2(__uint_as_float(sr[64 * h + 2 * i]), __uint_as_float(sr[64 * h + 2 * i + 1])),
-                                sc2, nm2);
+                        for (int i = 0; i < 16; ++i) {
+                            const int c = 32 * h + 2 * i;
+                            const float2 x = __ffma2_rn(make_float2(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])),
+                                                        sc2, nm2);
                             const float2 pp = make_float2(ex2_approx(x.x), ex2_approx(x.y));
                             ls[i & 1] = __fadd2_rn(ls[i & 1], pp);
-                            pk[i] = pack_bf16x2(pp.x, pp.y);
+                            pk[16 * h + i] = pack_bf16x2(pp.x, pp.y);
                         }
-                        tmem_st32(trow + scol + 32 * h, pk);
+                        tmem_st16_async(trow + scol + 16 * h, &pk[16 * h]);
                     }
+                    tmem_wait_st();
                     l_run += (ls[0].x + ls[1].x) + (ls[0].y + ls[1].y);
                     if (warp_need) {
                         // PV of the previous block has completed: this block's S was issued after it

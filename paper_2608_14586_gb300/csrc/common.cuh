@@ -115,6 +115,23 @@ VLA_DEV void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_
                  : "memory");
 }
 
+// 2-D TMA tile store shared memory -> global (x innermost); out-of-range parts of the box are
+// not written. Completion is tracked with bulk async-groups of the issuing thread.
+VLA_DEV void tma_store_2d(const CUtensorMap* map, const void* smem_src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(smem_u32(smem_src)), "r"(x), "r"(y)
+                 : "memory");
+}
+VLA_DEV void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// wait until at most N of this thread's bulk groups still read their shared-memory source
+template <int N>
+VLA_DEV void bulk_wait_group_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// wait until all of this thread's bulk groups have completed (writes performed)
+VLA_DEV void bulk_wait_group_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // named barrier over `count` threads (a subset of the CTA), id 1..15
 VLA_DEV void named_sync(int id, int count) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory"); }
 
@@ -258,6 +275,18 @@ VLA_DEV void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
         "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
         : "memory");
 }
+
+// 32 lanes x 16 consecutive 32-bit columns to TMEM, not waited on: the source registers stay
+// in use until tmem_wait_st()
+VLA_DEV void tmem_st16_async(uint32_t taddr, const uint32_t* r) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};\n" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+VLA_DEV void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 // Shared-memory descriptor of an MN-major operand written by TMA with 128-byte swizzling:
 // rows along K of 64 MN-contiguous bf16 (128 B), 8-row swizzle atoms; `mn_stride` bytes

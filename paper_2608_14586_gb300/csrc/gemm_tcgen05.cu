@@ -31,15 +31,19 @@ constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kThreads = 192;
 
-template <int BN>
+template <int BN, int EPI>
 struct GemmCfg {
     static constexpr uint32_t A_BYTES = kBM * kBK * 2;
     static constexpr uint32_t B_BYTES = BN * kBK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    // as many stages as fit in 227 KB next to the alignment pad and barriers, at most 6
-    static constexpr int STAGES = (232448 - 1280) / STAGE_BYTES < 6 ? (232448 - 1280) / STAGE_BYTES : 6;
+    // residual epilogue: per epilogue warp two 32 x 32 bf16 staging boxes for its TMA stores
+    static constexpr uint32_t OUT_BYTES = EPI == kEpiResid ? 4 * 2 * 2048 : 0;
+    static constexpr uint32_t FIXED = 1024 /*align*/ + 1024 /*barriers, staging alignment*/ + OUT_BYTES;
+    // as many stages as fit in 227 KB next to the fixed part, at most 6
+    static constexpr int STAGES = (232448 - FIXED) / STAGE_BYTES < 6 ? (232448 - FIXED) / STAGE_BYTES : 6;
     static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;  // two accumulators, a power of two
-    static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+    static constexpr uint32_t OFF_OUT = STAGES * STAGE_BYTES + 1024;  // 1024-aligned
+    static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + FIXED;
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
 };
 
@@ -147,6 +151,71 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
     if (ep.ss_out && ep.ss_width == 256 && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_groups + n0 / 256] = ss;
 }
 
+// The same residual epilogue with the stores made by TMA: each 32-column chunk of the warp's
+// 32 rows is packed into a 32 x 32 bf16 box in shared memory (64-byte swizzle, so the 16-byte
+// writes of the 32 lanes spread over all banks) and one lane stores the box with
+// cp.async.bulk.tensor; the box rows past M and columns past N are clipped by the tensor map.
+// Two boxes per warp alternate, the older store's read of its box waited for before reuse.
+// Needs N a multiple of 32 and no host copy (out_host). Row statistics as epi_plain_resid.
+template <int BN>
+VLA_DEV void epi_resid_tma(uint32_t taddr, int row, int row0, int n0, const EpiParams& ep, const CUtensorMap* tm_out,
+                           uint8_t* stage, uint32_t& nstore, int lane) {
+    const bool row_ok = row < ep.M;
+    float ss = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        const int col = n0 + c;
+        if (col >= ep.N) continue;  // uniform over the warp
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
+        if (row_ok && ep.resid) {
+            const uint4* rp = reinterpret_cast<const uint4*>(ep.resid + (size_t)row * ep.ld_resid + col);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                uint4 q = rp[i];
+                v[i * 8 + 0] += bf16_lo(q.x);
+                v[i * 8 + 1] += bf16_hi(q.x);
+                v[i * 8 + 2] += bf16_lo(q.y);
+                v[i * 8 + 3] += bf16_hi(q.y);
+                v[i * 8 + 4] += bf16_lo(q.z);
+                v[i * 8 + 5] += bf16_hi(q.z);
+                v[i * 8 + 6] += bf16_lo(q.w);
+                v[i * 8 + 7] += bf16_hi(q.w);
+            }
+        }
+        if (ep.ss_out && row_ok) {  // the group's sum of squares of the stored values, a chain from zero
+            float g = 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const float rr = __bfloat162float(__float2bfloat16_rn(v[i]));
+                g = fmaf(rr, rr, g);
+            }
+            if (ep.ss_width == 32) ep.ss_out[(size_t)row * ep.ss_groups + (col >> 5)] = g;
+            else ss += g;
+        }
+        uint8_t* box = stage + (nstore & 1u) * 2048u;
+        if (lane == 0) bulk_wait_group_read<1>();  // the store that last used this box has read it
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint4 o = make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+            *reinterpret_cast<uint4*>(box + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = o;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+            tma_store_2d(tm_out, box, col, row0);
+            bulk_commit_group();
+        }
+        ++nstore;
+    }
+    if (ep.ss_out && ep.ss_width == 256 && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_groups + n0 / 256] = ss;
+}
+
 VLA_DEV void store_bf16x16(bf16* dst, const float* v) {
     uint4* d = reinterpret_cast<uint4*>(dst);
 #pragma unroll
@@ -244,9 +313,9 @@ VLA_DEV bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_f
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M,
-                      int N, int K, EpiParams ep) {
-    using C = GemmCfg<BN>;
+    gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ CUtensorMap tmOut, int M, int N, int K, EpiParams ep) {
+    using C = GemmCfg<BN, EPI>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     __shared__ volatile int s_abort;
@@ -413,6 +482,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         pdl_trigger();
         const int quarter = warp & 3;  // TMEM lanes [32*quarter, 32*quarter + 32)
         int it = 0;
+        uint32_t nstore = 0;  // TMA stores of this warp (residual epilogue through TMA)
+        uint8_t* stage_out = smem + C::OFF_OUT + (uint32_t)(warp - 2) * 4096u;
         for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++it) {
             const int acc = it & 1;
             const uint32_t acc_phase = (it >> 1) & 1;
@@ -433,11 +504,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else if constexpr (EPI == kEpiSwiGLU) {
                 epi_swiglu<BN>(taddr, row, n0, ep);
             } else {
-                epi_plain_resid<BN>(taddr, row, n0, ep);
+                if (ep.tma_out) epi_resid_tma<BN>(taddr, row, m0 + quarter * 32, n0, ep, &tmOut, stage_out, nstore, lane);
+                else epi_plain_resid<BN>(taddr, row, n0, ep);
             }
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }
+        // the TMA stores of this warp are complete (their writes performed) before the CTA exits
+        if (EPI == kEpiResid && ep.tma_out && lane == 0) bulk_wait_group_all();
     }
     __syncwarp();
     tc_fence_before();
@@ -449,9 +523,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K, const EpiParams& ep,
-                       int num_sms, cudaStream_t stream, bool pdl) {
-    using C = GemmCfg<BN>;
+cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, const CUtensorMap& Out, int M, int N, int K,
+                       const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl) {
+    using C = GemmCfg<BN, EPI>;
     static bool attr_set = false;
     auto kern = gemm_bf16_tcgen05<BN, EPI>;
     if (!attr_set) {
@@ -461,27 +535,31 @@ cudaError_t launch_one(const CUtensorMap& A, const CUtensorMap& B, int M, int N,
     }
     const int tiles = ((M + kBM - 1) / kBM) * ((N + BN - 1) / BN);
     const int grid = tiles < num_sms ? tiles : num_sms;
-    return launch_ex(kern, dim3(grid), dim3(kThreads), C::SMEM_BYTES, stream, pdl, A, B, M, N, K, ep);
+    return launch_ex(kern, dim3(grid), dim3(kThreads), C::SMEM_BYTES, stream, pdl, A, B, Out, M, N, K, ep);
 }
 
 }  // namespace
 
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
-                        const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl) {
+                        const EpiParams& ep_in, int num_sms, cudaStream_t stream, bool pdl, const CUtensorMap* out_map) {
     if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
+    EpiParams ep = ep_in;
+    // residual / plain epilogue through TMA stores when an output map is given (no host copy)
+    ep.tma_out = (out_map && (mode == kEpiResid || mode == kEpiPlain) && !ep.out_host && N % 32 == 0) ? 1 : 0;
+    const CUtensorMap& O = ep.tma_out ? *out_map : A;  // unused unless tma_out
     if (bn == 256) {
         switch (mode) {
             case kEpiPlain:
-            case kEpiResid: return launch_one<256, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
-            case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
-            case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiResid: return launch_one<256, kEpiResid>(A, B, O, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiQKV: return launch_one<256, kEpiQKV>(A, B, O, M, N, K, ep, num_sms, stream, pdl);
+            case kEpiSwiGLU: return launch_one<256, kEpiSwiGLU>(A, B, O, M, N, K, ep, num_sms, stream, pdl);
         }
     } else if (bn == 224) {
         if (ep.ss_out && ep.ss_width != 32) return cudaErrorInvalidValue;  // partials would straddle tiles
         if (mode == kEpiResid || mode == kEpiPlain)
-            return launch_one<224, kEpiResid>(A, B, M, N, K, ep, num_sms, stream, pdl);
+            return launch_one<224, kEpiResid>(A, B, O, M, N, K, ep, num_sms, stream, pdl);
     } else if (bn == 192) {
-        if (mode == kEpiQKV) return launch_one<192, kEpiQKV>(A, B, M, N, K, ep, num_sms, stream, pdl);
+        if (mode == kEpiQKV) return launch_one<192, kEpiQKV>(A, B, O, M, N, K, ep, num_sms, stream, pdl);
     }
     return cudaErrorInvalidValue;
 }

@@ -76,6 +76,7 @@ struct EpiParams {
     // of each CTA's first tile is never loaded, so the waits on it run out (-1: no fault).
     long long wait_budget;
     int stall_kb;
+    int tma_out;  // set by launch_gemm: the residual epilogue stores through TMA
 };
 
 // Tensor-map helper (driver entry point fetched through the runtime). rows x cols bf16,
@@ -88,6 +89,10 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t 
 bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t rows, uint64_t planes,
                        uint64_t plane_stride, uint32_t box_rows);
 
+// Output map of a GEMM epilogue that stores through TMA: rows x cols bf16, row stride in
+// elements; box = 32 rows x 32 columns (64-byte rows), 64-byte swizzle.
+bool make_tmap_bf16_store(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride);
+
 // Programmatic dependent launch is used unless the environment sets VLA_NO_PDL (read once;
 // for profilers and debuggers that serialise kernels anyway).
 bool pdl_enabled();
@@ -96,8 +101,11 @@ bool pdl_enabled();
 // statistics then per 32 columns) or 192 (kEpiQKV). Returns a cudaError_t of the launch.
 // pdl: programmatic dependent launch (the CTA prologue and the first weight-tile loads may
 // overlap the previous kernel; A and everything the epilogue reads come after the wait).
+// out_map (optional, kEpiResid / kEpiPlain): the output as a make_tmap_bf16_store map; the
+// epilogue then stores through TMA (used when there is no host copy and N is a multiple of 32).
 cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMap& B, int M, int N, int K,
-                        const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl = false);
+                        const EpiParams& ep, int num_sms, cudaStream_t stream, bool pdl = false,
+                        const CUtensorMap* out_map = nullptr);
 
 // ---------------------------------------------------------------------------------------
 // Prefill attention (causal GQA, flash-style online softmax, attention_tc.cu)

@@ -78,6 +78,19 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t inner, uint6
     return r == CUDA_SUCCESS;
 }
 
+bool make_tmap_bf16_store(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride) {
+    PFN_encodeTiled_t enc = get_encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {row_stride * 2};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 bool pdl_enabled() {
     static const bool on = std::getenv("VLA_NO_PDL") == nullptr;
     return on;
@@ -508,6 +521,11 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         !vla::make_tmap_bf16(&tm_xmid, p->ws_xmid, M, D, D, 128) ||
         !vla::make_tmap_bf16(&tm_m, p->ws_m, M, p->F_pad, p->F_pad, 128))
         return VLA_ERR_CUDA;
+    // output maps of the O and down projections (epilogue stores through TMA)
+    CUtensorMap tm_st_xmid, tm_st_out;
+    if (!vla::make_tmap_bf16_store(&tm_st_xmid, p->ws_xmid, M, D, D) ||
+        !vla::make_tmap_bf16_store(&tm_st_out, hidden_out, M, D, D))
+        return VLA_ERR_CUDA;
     const float eps = p->cfg.rms_eps;
     int launches = 0;
     cudaError_t e = cudaSuccess;
@@ -606,7 +624,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         set_waits(p, eo, VLA_STAGE_GEMM_O, p->qc);
         stage_mark(p, VLA_STAGE_GEMM_O, true);
         e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_attn, d_bn == 224 ? ld.tm_o224 : ld.tm_o, M, D, p->qc, eo,
-                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_O));
+                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_O), &tm_st_xmid);
         stage_mark(p, VLA_STAGE_GEMM_O, false);
         if (e != cudaSuccess) break;
         // RMSNorm (row statistics from the O epilogue) + gate/up + SwiGLU
@@ -643,7 +661,7 @@ static vla_status prefill_impl(vla_prefix* p, const void* hidden_in, int n_token
         set_waits(p, ed, VLA_STAGE_GEMM_DOWN, p->F_pad);
         stage_mark(p, VLA_STAGE_GEMM_DOWN, true);
         e = vla::launch_gemm(vla::kEpiResid, d_bn, tm_m, d_bn == 224 ? ld.tm_d224 : ld.tm_d, M, D, p->F_pad, ed,
-                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_DOWN));
+                             p->num_sms, stream, pdl(VLA_STAGE_GEMM_DOWN), &tm_st_out);
         stage_mark(p, VLA_STAGE_GEMM_DOWN, false);
         launches += 5;
     }
@@ -909,7 +927,9 @@ vla_status vla_op_gemm_bf16(const void* A, const void* B, int M, int N, int K, v
     ep.ld_out = N;
     set_waits(nullptr, ep, -1, K);
     static const int sms = vla::device_sm_count();
-    return cuda_status(vla::launch_gemm(vla::kEpiPlain, kBN, ta, tb, M, N, K, ep, sms, (cudaStream_t)stream));
+    CUtensorMap tc;
+    if (!vla::make_tmap_bf16_store(&tc, C, M, N, N)) return VLA_ERR_CUDA;
+    return cuda_status(vla::launch_gemm(vla::kEpiPlain, kBN, ta, tb, M, N, K, ep, sms, (cudaStream_t)stream, false, &tc));
 }
 
 vla_status vla_op_attention_prefill(const void* q, const void* k_plane, const void* v_plane, int n_tokens,
