@@ -36,8 +36,9 @@ struct GemmCfg {
     static constexpr uint32_t A_BYTES = kBM * kBK * 2;
     static constexpr uint32_t B_BYTES = BN * kBK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-    // residual epilogue: per epilogue warp two 32 x 32 bf16 staging boxes for its TMA stores
-    static constexpr uint32_t OUT_BYTES = EPI == kEpiResid ? 4 * 2 * 2048 : 0;
+    // residual epilogue at 256-column tiles: per epilogue warp two 32 x 32 bf16 staging boxes
+    // for its TMA stores (224-column tiles keep their fifth stage and store directly)
+    static constexpr uint32_t OUT_BYTES = (EPI == kEpiResid && BN == 256) ? 4 * 2 * 2048 : 0;
     static constexpr uint32_t FIXED = 1024 /*align*/ + 1024 /*barriers, staging alignment*/ + OUT_BYTES;
     // as many stages as fit in 227 KB next to the fixed part, at most 6
     static constexpr int STAGES = (232448 - FIXED) / STAGE_BYTES < 6 ? (232448 - FIXED) / STAGE_BYTES : 6;
@@ -160,22 +161,36 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
 template <int BN>
 VLA_DEV void epi_resid_tma(uint32_t taddr, int row, int row0, int n0, const EpiParams& ep, const CUtensorMap* tm_out,
                            uint8_t* stage, uint32_t& nstore, int lane) {
+    constexpr int NC = BN / 32;
     const bool row_ok = row < ep.M;
+    const bool has_res = row_ok && ep.resid != nullptr;
+    const uint4* rrow = has_res ? reinterpret_cast<const uint4*>(ep.resid + (size_t)row * ep.ld_resid + n0) : nullptr;
+    // the residual chunks are requested two ahead of their use, so their latency overlaps the
+    // tensor-memory reads and the stores of the chunks before
+    uint4 res[3][4];
+    auto fetch = [&](int c) {
+        if (has_res && n0 + 32 * c < ep.N) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) res[c % 3][i] = rrow[4 * c + i];
+        }
+    };
+    fetch(0);
+    if (NC > 1) fetch(1);
     float ss = 0.f;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
+#pragma unroll
+    for (int c = 0; c < NC; ++c) {
+        if (c + 2 < NC) fetch(c + 2);
         uint32_t r[32];
-        tmem_ld32(taddr + c, r);
-        const int col = n0 + c;
+        tmem_ld32(taddr + 32 * c, r);
+        const int col = n0 + 32 * c;
         if (col >= ep.N) continue;  // uniform over the warp
         float v[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
-        if (row_ok && ep.resid) {
-            const uint4* rp = reinterpret_cast<const uint4*>(ep.resid + (size_t)row * ep.ld_resid + col);
+        if (has_res) {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                uint4 q = rp[i];
+                const uint4 q = res[c % 3][i];
                 v[i * 8 + 0] += bf16_lo(q.x);
                 v[i * 8 + 1] += bf16_hi(q.x);
                 v[i * 8 + 2] += bf16_lo(q.y);
@@ -504,14 +519,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else if constexpr (EPI == kEpiSwiGLU) {
                 epi_swiglu<BN>(taddr, row, n0, ep);
             } else {
-                if (ep.tma_out) epi_resid_tma<BN>(taddr, row, m0 + quarter * 32, n0, ep, &tmOut, stage_out, nstore, lane);
-                else epi_plain_resid<BN>(taddr, row, n0, ep);
+                if (C::OUT_BYTES && ep.tma_out)
+                    epi_resid_tma<BN>(taddr, row, m0 + quarter * 32, n0, ep, &tmOut, stage_out, nstore, lane);
+                else
+                    epi_plain_resid<BN>(taddr, row, n0, ep);
             }
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
         }
         // the TMA stores of this warp are complete (their writes performed) before the CTA exits
-        if (EPI == kEpiResid && ep.tma_out && lane == 0) bulk_wait_group_all();
+        if (C::OUT_BYTES && ep.tma_out && lane == 0) bulk_wait_group_all();
     }
     __syncwarp();
     tc_fence_before();
@@ -545,7 +562,8 @@ cudaError_t launch_gemm(int mode, int bn, const CUtensorMap& A, const CUtensorMa
     if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
     EpiParams ep = ep_in;
     // residual / plain epilogue through TMA stores when an output map is given (no host copy)
-    ep.tma_out = (out_map && (mode == kEpiResid || mode == kEpiPlain) && !ep.out_host && N % 32 == 0) ? 1 : 0;
+    ep.tma_out =
+        (out_map && bn == 256 && (mode == kEpiResid || mode == kEpiPlain) && !ep.out_host && N % 32 == 0) ? 1 : 0;
     const CUtensorMap& O = ep.tma_out ? *out_map : A;  // unused unless tma_out
     if (bn == 256) {
         switch (mode) {
