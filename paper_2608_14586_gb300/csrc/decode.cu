@@ -125,16 +125,23 @@ VLA_DEV void gemv_epilogue(const GemvParams& p, int b, int u, int ra, int rb, fl
     }
 }
 
-template <int MODE, int NB>
+// KS = 1: one warp per row pair. KS = 2: two warps of a CTA per row pair, each over half of
+// K; the second half's sums reach the first warp through shared memory behind a 64-thread
+// named barrier and are added in that fixed order (used where the row pairs would otherwise
+// leave a mostly idle last round of warps: the QKV projection's 3072 pairs on 2432 warps).
+template <int MODE, int NB, int KS>
 __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_constant__ GemvParams p) {
     extern __shared__ uint4 xs[];  // [NB][K/8]
     __shared__ float red[NB][kGemvThreads / 32];
     __shared__ float s_rinv[NB];
+    __shared__ float s_half[kGemvThreads / 64][2][NB][2];  // KS = 2: [warp pair][unit parity][b][a, b]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int gw = blockIdx.x * (kGemvThreads / 32) + warp;
-    const int nw = gridDim.x * (kGemvThreads / 32);
-    const int nchunk = p.K >> 3;        // 16-byte chunks per row
-    const int nstep = nchunk >> 5;      // chunk steps of the whole warp
+    const int gw = (blockIdx.x * (kGemvThreads / 32) + warp) / KS;  // the warp's (pair's) unit slot
+    const int hk = KS == 2 ? (warp & 1) : 0;                         // which half of K
+    const int nw = gridDim.x * (kGemvThreads / 32) / KS;
+    const int nchunk = p.K >> 3;          // 16-byte chunks per row
+    const int nstep = (nchunk >> 5) / KS; // chunk steps of the warp over its share of K
+    const int s_base = hk * nstep;        // first chunk step of this warp
 
     // Weights do not depend on the previous kernel. Under programmatic dependent launch this
     // part runs while the previous kernel drains: warm L2 with this warp's first row pair and
@@ -144,9 +151,9 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_cons
     if (gw < p.units) {
         int ra, rb;
         unit_rows<MODE>(p, gw, ra, rb);
-        const char* pa = reinterpret_cast<const char*>(p.W + (size_t)ra * p.K);
-        const char* pb = reinterpret_cast<const char*>(p.W + (size_t)rb * p.K);
-        for (int l = lane; l < (p.K * 2) / 128; l += 32) {
+        const char* pa = reinterpret_cast<const char*>(p.W + (size_t)ra * p.K) + (size_t)s_base * 512;
+        const char* pb = reinterpret_cast<const char*>(p.W + (size_t)rb * p.K) + (size_t)s_base * 512;
+        for (int l = lane; l < (p.K * 2 / KS) / 128; l += 32) {
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pa + l * 128));
             asm volatile("prefetch.global.L2 [%0];" ::"l"(pb + l * 128));
         }
@@ -198,11 +205,13 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_cons
         for (int b = 0; b < NB; ++b) pos[b] = *p.d_len[b];
     }
 
-    for (int u = gw; u < p.units; u += nw) {
+    int k = 0;  // units done by this warp (KS = 2: the exchange slot's parity)
+    for (int u = gw; u < p.units; u += nw, ++k) {
         int ra, rb;
         unit_rows<MODE>(p, u, ra, rb);
-        const uint4* wa = reinterpret_cast<const uint4*>(p.W + (size_t)ra * p.K);
-        const uint4* wb = reinterpret_cast<const uint4*>(p.W + (size_t)rb * p.K);
+        const uint4* wa = reinterpret_cast<const uint4*>(p.W + (size_t)ra * p.K) + s_base * 32;
+        const uint4* wb = reinterpret_cast<const uint4*>(p.W + (size_t)rb * p.K) + s_base * 32;
+        const uint4* xk = xs + s_base * 32;
         float acc_a[NB], acc_b[NB];
 #pragma unroll
         for (int b = 0; b < NB; ++b) acc_a[b] = acc_b[b] = 0.f;
@@ -220,19 +229,40 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_cons
                 if (s + i < nstep) {
 #pragma unroll
                     for (int b = 0; b < NB; ++b) {
-                        const uint4 x = xs[b * nchunk + (s + i) * 32 + lane];
+                        const uint4 x = xk[b * nchunk + (s + i) * 32 + lane];
                         acc_a[b] += dot8(va[i], x);
                         acc_b[b] += dot8(vb[i], x);
                     }
                 }
             }
         }
+        float sa[NB], sb[NB];
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
-            const float sa = warp_sum(acc_a[b]);
-            const float sb = warp_sum(acc_b[b]);
-            if (lane == 0) gemv_epilogue<MODE>(p, b, u, ra, rb, sa, sb, rinv[b], pos[b]);
+            sa[b] = warp_sum(acc_a[b]);
+            sb[b] = warp_sum(acc_b[b]);
         }
+        if constexpr (KS == 2) {
+            // both warps of the pair run the same units, so they meet here the same number of times
+            float(&slot)[NB][2] = s_half[warp >> 1][k & 1];
+            if (hk == 1 && lane == 0) {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    slot[b][0] = sa[b];
+                    slot[b][1] = sb[b];
+                }
+            }
+            named_sync(1 + (warp >> 1), 64);
+            if (hk == 1) continue;
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                sa[b] += slot[b][0];
+                sb[b] += slot[b][1];
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+            if (lane == 0) gemv_epilogue<MODE>(p, b, u, ra, rb, sa[b], sb[b], rinv[b], pos[b]);
     }
 }
 
@@ -476,21 +506,37 @@ __global__ void advance_lengths_kernel(const __grid_constant__ LenPtrs lp, int c
     if (i < count) lp.p[blockIdx.x][i] += 1;
 }
 
-template <int MODE, int NB>
-cudaError_t launch_gemv_nb(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
+template <int MODE, int NB, int KS>
+cudaError_t launch_gemv_ks(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
+    auto kern = gemv_kernel<MODE, NB, KS>;
     const size_t smem = (size_t)NB * p.K * 2;
     static size_t attr = 0;
     if (smem > attr) {
-        cudaError_t e =
-            cudaFuncSetAttribute(gemv_kernel<MODE, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         attr = smem;
     }
-    const int warps_needed = p.units;
-    int grid = 2 * num_sms;
-    const int gmax = (warps_needed + 7) / 8;
-    if (grid > gmax) grid = gmax;
-    return launch_ex(gemv_kernel<MODE, NB>, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
+    int grid;
+    if (KS == 1) {
+        grid = 2 * num_sms;
+        const int gmax = (p.units + 7) / 8;
+        if (grid > gmax) grid = gmax;
+    } else {
+        // as few rounds of row pairs per warp pair as the resident warps allow (two CTAs per
+        // SM), then as few CTAs as that round count needs, so every pair gets the same number
+        const int slots_max = 2 * num_sms * (kGemvThreads / 32) / KS;
+        const int rounds = (p.units + slots_max - 1) / slots_max;
+        const int slots = (p.units + rounds - 1) / rounds;
+        grid = (slots * KS + (kGemvThreads / 32) - 1) / (kGemvThreads / 32);
+    }
+    return launch_ex(kern, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
+}
+
+template <int MODE, int NB>
+cudaError_t launch_gemv_nb(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
+    // the QKV projection splits K over two warps per row pair (K a multiple of 512)
+    if (MODE == kGemvQKV && p.K % 512 == 0) return launch_gemv_ks<MODE, NB, 2>(p, num_sms, s, pdl);
+    return launch_gemv_ks<MODE, NB, 1>(p, num_sms, s, pdl);
 }
 
 template <int MODE>
