@@ -316,6 +316,10 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) {
 VLA_DEV void cluster_sync_all() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// Split form of the same barrier: a relaxed arrival early in the kernel and the wait before
+// the first distributed-shared-memory access guarantee that every CTA of the cluster runs.
+VLA_DEV void cluster_arrive_relaxed() { asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory"); }
+VLA_DEV void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
 // 32-bit store into the same shared-memory variable in CTA `rank` of the cluster
 VLA_DEV void st_dsmem_f32(float* local, uint32_t rank, float v) {
     uint32_t remote;

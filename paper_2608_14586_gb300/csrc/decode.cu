@@ -2,8 +2,10 @@
 //
 // At M = 1 every projection is a matrix-vector product whose cost is streaming the weights
 // once from HBM (354 MB per 7B-class block), so these kernels are built for bandwidth:
-//   * one warp per pair of weight rows, 16-byte non-allocating loads, 8 chunks per row in
-//     flight per lane, fp32 FMA, warp-shuffle reduction;
+//   * each warp takes a contiguous range of row pairs (the same count for every warp) and
+//     streams their rows through a ring of shared-memory slots with 1-D bulk copies
+//     (cp.async.bulk, completion on per-slot mbarriers), up to 24 KB per warp and 192 KB per
+//     SM in flight; fp32 FMA over 16-byte chunks, warp-shuffle reduction;
 //   * the pair is chosen so the fused epilogue has both operands it needs: dims (j, j+dh/2)
 //     of a head for the rotary embedding (adjacent rows of the repacked q/k weights), the
 //     gate and up rows of one feed-forward unit for SwiGLU, consecutive rows for the
@@ -11,8 +13,8 @@
 //   * the input vector is staged in shared memory; RMSNorm's 1/rms is computed per CTA
 //     (the gains are folded into the weights);
 //   * under programmatic dependent launch each kernel starts while its predecessor drains:
-//     it prefetches its first weight rows into L2 and loads the first batch into registers,
-//     and reads nothing that an earlier kernel of the step wrote before griddepcontrol.wait.
+//     it requests the first ring slots of its weight rows, and reads nothing that an earlier
+//     kernel of the step wrote before griddepcontrol.wait.
 // Attention is split over the context inside one thread-block cluster per KV head (16 CTAs
 // where the device schedules such clusters, else 8; fixed split count -> deterministic): each
 // CTA bulk-copies its contiguous key range of K and V into shared memory (the rows that
@@ -47,10 +49,15 @@ struct GemvParams {
     const float2* rope;
     int dh, n_q_heads, n_kv_heads, max_ctx;
     float eps;
+    unsigned* status;  // timeout report (a weight copy that never lands)
+    int per_warp;      // row pairs per warp (set at launch)
+    int stages;        // ring slots per warp (set at launch)
 };
 
 constexpr int kGemvThreads = 256;
-constexpr int kGemvU = 8;  // 16-byte chunks per row in flight per lane
+constexpr int kGemvWarps = kGemvThreads / 32;
+constexpr int kGemvSegBytes = 4096;  // bytes of each row per ring slot
+constexpr int kGemvMaxStages = 3;
 
 VLA_DEV float dot8(uint4 w, uint4 x) {
     float a = bf16_lo(w.x) * bf16_lo(x.x);
@@ -125,53 +132,53 @@ VLA_DEV void gemv_epilogue(const GemvParams& p, int b, int u, int ra, int rb, fl
     }
 }
 
-// KS = 1: one warp per row pair. KS = 2: two warps of a CTA per row pair, each over half of
-// K; the second half's sums reach the first warp through shared memory behind a 64-thread
-// named barrier and are added in that fixed order (used where the row pairs would otherwise
-// leave a mostly idle last round of warps: the QKV projection's 3072 pairs on 2432 warps).
-template <int MODE, int NB, int KS>
-__global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_constant__ GemvParams p) {
-    extern __shared__ uint4 xs[];  // [NB][K/8]
-    __shared__ float red[NB][kGemvThreads / 32];
+// One warp per contiguous range of `per_warp` row pairs (balanced: every warp but the last
+// takes the same count, and the grid has as many CTAs as that needs, at most one per SM).
+// Lane 0 of each warp streams its pairs' rows through the warp's ring of `stages` slots, each
+// slot a 4 KB segment of both rows of a pair, with 1-D bulk copies completing on the slot's
+// mbarrier; the first slots are requested before griddepcontrol.wait, since the weights do
+// not depend on the previous kernel. Lane l accumulates the 16-byte chunks l, l + 32, ... of
+// the row in order (fp32), then the warp reduces and lane 0 applies the fused epilogue.
+template <int MODE, int NB>
+__global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const __grid_constant__ GemvParams p) {
+    extern __shared__ __align__(16) uint8_t gsm[];
+    uint4* xs = reinterpret_cast<uint4*>(gsm);  // [NB][K/8] input vectors
+    __shared__ uint64_t full[kGemvWarps][kGemvMaxStages];
+    __shared__ float red[NB][kGemvWarps];
     __shared__ float s_rinv[NB];
-    __shared__ float s_half[kGemvThreads / 64][2][NB][2];  // KS = 2: [warp pair][unit parity][b][a, b]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int gw = (blockIdx.x * (kGemvThreads / 32) + warp) / KS;  // the warp's (pair's) unit slot
-    const int hk = KS == 2 ? (warp & 1) : 0;                         // which half of K
-    const int nw = gridDim.x * (kGemvThreads / 32) / KS;
-    const int nchunk = p.K >> 3;          // 16-byte chunks per row
-    const int nstep = (nchunk >> 5) / KS; // chunk steps of the warp over its share of K
-    const int s_base = hk * nstep;        // first chunk step of this warp
+    const int gw = blockIdx.x * kGemvWarps + warp;
+    const int nchunk = p.K >> 3;  // 16-byte chunks per row
+    const int row_bytes = p.K * 2;
+    const int nseg = (row_bytes + kGemvSegBytes - 1) / kGemvSegBytes;
+    const int u0 = gw * p.per_warp;
+    const int T = max(0, min(p.units, u0 + p.per_warp) - u0) * nseg;  // ring stages of this warp
+    const int S = p.stages;
+    uint8_t* ring = gsm + (size_t)NB * row_bytes + (size_t)warp * S * 2 * kGemvSegBytes;
 
-    // Weights do not depend on the previous kernel. Under programmatic dependent launch this
-    // part runs while the previous kernel drains: warm L2 with this warp's first row pair and
-    // load its first batch of chunks into registers. Nothing written by an earlier kernel is
-    // read before pdl_wait().
-    uint4 va[kGemvU], vb[kGemvU];
-    if (gw < p.units) {
+    // lane 0: segment t % nseg of row pair u0 + t / nseg into slot t % S
+    auto issue = [&](int t) {
+        const int u = u0 + t / nseg, sg = t % nseg;
         int ra, rb;
-        unit_rows<MODE>(p, gw, ra, rb);
-        const char* pa = reinterpret_cast<const char*>(p.W + (size_t)ra * p.K) + (size_t)s_base * 512;
-        const char* pb = reinterpret_cast<const char*>(p.W + (size_t)rb * p.K) + (size_t)s_base * 512;
-        for (int l = lane; l < (p.K * 2 / KS) / 128; l += 32) {
-            asm volatile("prefetch.global.L2 [%0];" ::"l"(pa + l * 128));
-            asm volatile("prefetch.global.L2 [%0];" ::"l"(pb + l * 128));
-        }
-        const uint4* wa = reinterpret_cast<const uint4*>(pa);
-        const uint4* wb = reinterpret_cast<const uint4*>(pb);
-#pragma unroll
-        for (int i = 0; i < kGemvU; ++i) {
-            if (i < nstep) {
-                va[i] = ldg_stream(wa + i * 32 + lane);
-                vb[i] = ldg_stream(wb + i * 32 + lane);
-            }
-        }
+        unit_rows<MODE>(p, u, ra, rb);
+        const int off = sg * kGemvSegBytes;
+        const uint32_t bytes = (uint32_t)min(kGemvSegBytes, row_bytes - off);
+        uint64_t* bar = &full[warp][t % S];
+        uint8_t* dst = ring + (size_t)(t % S) * 2 * kGemvSegBytes;
+        mbar_arrive_expect_tx(bar, 2 * bytes);
+        bulk_load(dst, reinterpret_cast<const uint8_t*>(p.W + (size_t)ra * p.K) + off, bytes, bar);
+        bulk_load(dst + kGemvSegBytes, reinterpret_cast<const uint8_t*>(p.W + (size_t)rb * p.K) + off, bytes, bar);
+    };
+    if (lane == 0) {
+        for (int j = 0; j < S; ++j) mbar_init(&full[warp][j], 1);
+        fence_barrier_init();
+        for (int t = 0; t < min(T, S); ++t) issue(t);
     }
     pdl_wait();
     pdl_trigger();
     const uint4* xg = reinterpret_cast<const uint4*>(p.xv);
     for (int i = threadIdx.x; i < NB * nchunk; i += kGemvThreads) xs[i] = __ldcg(xg + i);
-    __syncthreads();
+    __syncthreads();  // also publishes the barrier initialisation to the whole warp
     float rinv[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) rinv[b] = 1.f;
@@ -189,7 +196,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_cons
         __syncthreads();
         if (threadIdx.x < NB) {
             float t = 0.f;
-            for (int w = 0; w < kGemvThreads / 32; ++w) t += red[threadIdx.x][w];
+            for (int w = 0; w < kGemvWarps; ++w) t += red[threadIdx.x][w];
             s_rinv[threadIdx.x] = 1.0f / sqrtf(t / (float)p.K + p.eps);
         }
         __syncthreads();
@@ -205,64 +212,53 @@ __global__ void __launch_bounds__(kGemvThreads, 2) gemv_kernel(const __grid_cons
         for (int b = 0; b < NB; ++b) pos[b] = *p.d_len[b];
     }
 
-    int k = 0;  // units done by this warp (KS = 2: the exchange slot's parity)
-    for (int u = gw; u < p.units; u += nw, ++k) {
-        int ra, rb;
-        unit_rows<MODE>(p, u, ra, rb);
-        const uint4* wa = reinterpret_cast<const uint4*>(p.W + (size_t)ra * p.K) + s_base * 32;
-        const uint4* wb = reinterpret_cast<const uint4*>(p.W + (size_t)rb * p.K) + s_base * 32;
-        const uint4* xk = xs + s_base * 32;
-        float acc_a[NB], acc_b[NB];
+    float acc_a[NB], acc_b[NB];
 #pragma unroll
-        for (int b = 0; b < NB; ++b) acc_a[b] = acc_b[b] = 0.f;
-        for (int s = 0; s < nstep; s += kGemvU) {
-#pragma unroll
-            for (int i = 0; i < kGemvU; ++i) {
-                if (s + i < nstep && (s > 0 || u != gw)) {  // batch 0 of the first unit is preloaded
-                    const int c = (s + i) * 32 + lane;
-                    va[i] = ldg_stream(wa + c);
-                    vb[i] = ldg_stream(wb + c);
-                }
-            }
-#pragma unroll
-            for (int i = 0; i < kGemvU; ++i) {
-                if (s + i < nstep) {
-#pragma unroll
-                    for (int b = 0; b < NB; ++b) {
-                        const uint4 x = xk[b * nchunk + (s + i) * 32 + lane];
-                        acc_a[b] += dot8(va[i], x);
-                        acc_b[b] += dot8(vb[i], x);
-                    }
-                }
-            }
-        }
-        float sa[NB], sb[NB];
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            sa[b] = warp_sum(acc_a[b]);
-            sb[b] = warp_sum(acc_b[b]);
-        }
-        if constexpr (KS == 2) {
-            // both warps of the pair run the same units, so they meet here the same number of times
-            float(&slot)[NB][2] = s_half[warp >> 1][k & 1];
-            if (hk == 1 && lane == 0) {
-#pragma unroll
-                for (int b = 0; b < NB; ++b) {
-                    slot[b][0] = sa[b];
-                    slot[b][1] = sb[b];
-                }
-            }
-            named_sync(1 + (warp >> 1), 64);
-            if (hk == 1) continue;
+    for (int b = 0; b < NB; ++b) acc_a[b] = acc_b[b] = 0.f;
+    int t = 0;
+    for (; t < T; ++t) {
+        const int slot = t % S, sg = t % nseg;
+        if (!__all_sync(0xFFFFFFFFu, mbar_wait(&full[warp][slot], (uint32_t)(t / S) & 1u))) break;
+        const uint4* wa = reinterpret_cast<const uint4*>(ring + (size_t)slot * 2 * kGemvSegBytes);
+        const uint4* wb = wa + kGemvSegBytes / 16;
+        const int c0 = sg * (kGemvSegBytes / 16);                       // first chunk of the segment
+        const int nch = min(kGemvSegBytes, row_bytes - sg * kGemvSegBytes) >> 4;  // a multiple of 32
+#pragma unroll 4
+        for (int c = lane; c < nch; c += 32) {
+            const uint4 va = wa[c], vb = wb[c];
 #pragma unroll
             for (int b = 0; b < NB; ++b) {
-                sa[b] += slot[b][0];
-                sb[b] += slot[b][1];
+                const uint4 x = xs[b * nchunk + c0 + c];
+                acc_a[b] += dot8(va, x);
+                acc_b[b] += dot8(vb, x);
             }
         }
+        __syncwarp();  // every lane has read the slot
+        if (lane == 0 && t + S < T) {
+            fence_proxy_async_smem();
+            issue(t + S);
+        }
+        if (sg == nseg - 1) {
+            const int u = u0 + t / nseg;
+            int ra, rb;
+            unit_rows<MODE>(p, u, ra, rb);
 #pragma unroll
-        for (int b = 0; b < NB; ++b)
-            if (lane == 0) gemv_epilogue<MODE>(p, b, u, ra, rb, sa[b], sb[b], rinv[b], pos[b]);
+            for (int b = 0; b < NB; ++b) {
+                const float sa = warp_sum(acc_a[b]);
+                const float sb = warp_sum(acc_b[b]);
+                if (lane == 0) gemv_epilogue<MODE>(p, b, u, ra, rb, sa, sb, rinv[b], pos[b]);
+                acc_a[b] = acc_b[b] = 0.f;
+            }
+        }
+    }
+    if (t < T) {
+        // a copy did not land within the wait budget: report it and let the copies already
+        // requested into this warp's ring finish (again bounded) before the CTA exits
+        if (lane == 0) {
+            set_status(p.status, kDevTimeout);
+            for (int r = t; r < min(T, t + S); ++r) mbar_wait(&full[warp][r % S], (uint32_t)(r / S) & 1u);
+        }
+        __syncwarp();
     }
 }
 
@@ -506,37 +502,25 @@ __global__ void advance_lengths_kernel(const __grid_constant__ LenPtrs lp, int c
     if (i < count) lp.p[blockIdx.x][i] += 1;
 }
 
-template <int MODE, int NB, int KS>
-cudaError_t launch_gemv_ks(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
-    auto kern = gemv_kernel<MODE, NB, KS>;
-    const size_t smem = (size_t)NB * p.K * 2;
+template <int MODE, int NB>
+cudaError_t launch_gemv_nb(const GemvParams& p_in, int num_sms, cudaStream_t s, bool pdl) {
+    GemvParams p = p_in;
+    if (p.K % 256 != 0 || p.units <= 0) return cudaErrorInvalidValue;
+    p.stages = NB == 1 ? 3 : 2;  // ring slots per warp within the shared memory of one CTA per SM
+    const size_t smem = (size_t)NB * p.K * 2 + (size_t)kGemvWarps * p.stages * 2 * kGemvSegBytes;
+    auto kern = gemv_kernel<MODE, NB>;
     static size_t attr = 0;
     if (smem > attr) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         attr = smem;
     }
-    int grid;
-    if (KS == 1) {
-        grid = 2 * num_sms;
-        const int gmax = (p.units + 7) / 8;
-        if (grid > gmax) grid = gmax;
-    } else {
-        // as few rounds of row pairs per warp pair as the resident warps allow (two CTAs per
-        // SM), then as few CTAs as that round count needs, so every pair gets the same number
-        const int slots_max = 2 * num_sms * (kGemvThreads / 32) / KS;
-        const int rounds = (p.units + slots_max - 1) / slots_max;
-        const int slots = (p.units + rounds - 1) / rounds;
-        grid = (slots * KS + (kGemvThreads / 32) - 1) / (kGemvThreads / 32);
-    }
+    // as few row pairs per warp as one CTA per SM allows, then as few warps as that count needs
+    const int max_warps = num_sms * kGemvWarps;
+    p.per_warp = (p.units + max_warps - 1) / max_warps;
+    const int warps = (p.units + p.per_warp - 1) / p.per_warp;
+    const int grid = (warps + kGemvWarps - 1) / kGemvWarps;
     return launch_ex(kern, dim3(grid), dim3(kGemvThreads), smem, s, pdl, p);
-}
-
-template <int MODE, int NB>
-cudaError_t launch_gemv_nb(const GemvParams& p, int num_sms, cudaStream_t s, bool pdl) {
-    // the QKV projection splits K over two warps per row pair (K a multiple of 512)
-    if (MODE == kGemvQKV && p.K % 512 == 0) return launch_gemv_ks<MODE, NB, 2>(p, num_sms, s, pdl);
-    return launch_gemv_ks<MODE, NB, 1>(p, num_sms, s, pdl);
 }
 
 template <int MODE>
@@ -695,6 +679,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     g.n_kv_heads = d.Hkv;
     g.max_ctx = d.max_ctx;
     g.eps = d.eps;
+    g.status = w.status;
     hook(kStageDecQKV, true);
     e = launch_gemv<kGemvQKV>(g, L.nb, num_sms, stream, pdl_first);
     hook(kStageDecQKV, false);
@@ -755,6 +740,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     o.xv = w.attn;
     o.resid = x_in;
     o.out = w.x_mid;
+    o.status = w.status;
     hook(kStageDecO, true);
     e = launch_gemv<kGemvResid>(o, L.nb, num_sms, stream, pdl);
     hook(kStageDecO, false);
@@ -767,6 +753,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     gu.xv = w.x_mid;
     gu.out = w.m;
     gu.eps = d.eps;
+    gu.status = w.status;
     hook(kStageDecGateUp, true);
     e = launch_gemv<kGemvSwiGLU>(gu, L.nb, num_sms, stream, pdl);
     hook(kStageDecGateUp, false);
@@ -779,6 +766,7 @@ cudaError_t launch_decode_layer(const DecodeLayer& L, const DecodeDims& d, const
     dn.xv = w.m;
     dn.resid = w.x_mid;
     dn.out = x_out;
+    dn.status = w.status;
     hook(kStageDecDown, true);
     e = launch_gemv<kGemvResid>(dn, L.nb, num_sms, stream, pdl);
     hook(kStageDecDown, false);

@@ -71,8 +71,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ uint64_t bar_kv, bar_mma;
     __shared__ uint32_t tmem_slot;
     __shared__ float red_m[4][G], red_l[4][G];
-    __shared__ float c_m[G], c_l[G];
-    __shared__ __align__(16) float c_o[G * kDH];
     // merge inbox: from each rank of the cluster, its (max, sum) per head and its unnormalised
     // output over this CTA's element slice
     __shared__ float rx_m[kMaxCs][G], rx_l[kMaxCs][G];
@@ -101,15 +99,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nbox = (nk + kBoxRows - 1) / kBoxRows;
     const int new_row = ctx - 1 - kb;  // slot of the token written by the QKV kernel
 
-    if (tid == 0) {
-        mbar_init(&bar_kv, 1);
-        mbar_init(&bar_mma, 1);
-        fence_barrier_init();
-        s_ok = 1;
-        tma_prefetch_desc(tmK);
-        tma_prefetch_desc(tmV);
-    }
+    // warp 0 requests the range's K and V rows that predate this step first: the copy is the
+    // longest part of the kernel when its CTAs start only as the QKV kernel's CTAs leave
     if (warp == 0) {
+        if (lane == 0) {
+            mbar_init(&bar_kv, 1);
+            mbar_init(&bar_mma, 1);
+            fence_barrier_init();
+            s_ok = 1;
+            mbar_arrive_expect_tx(&bar_kv, (uint32_t)nbox * 4u * kBoxBytes);
+        }
+        __syncwarp();
+        // lane l issues the copies (box b, d_h half c) = l, l + 32, ...
+        for (int i = lane; i < nbox * 2; i += 32) {
+            const int b = i >> 1, c = i & 1;
+            const int y = kb + b * kBoxRows;
+            const uint32_t dst = half_off(p.rows, b >> 2, c) + (uint32_t)(b & 3) * kBoxBytes;
+            tma_load_3d(sK + dst, tmK, &bar_kv, c * 64, y, kvh);
+            tma_load_3d(sV + dst, tmV, &bar_kv, c * 64, y, kvh);
+        }
+    }
+    pdl_wait();
+    pdl_trigger();
+
+    // global reads of what the QKV kernel wrote (Q and the new token's K and V rows) go out
+    // first; tensor memory and the zeroing of the Q and P tiles overlap their latency
+    const bool has_new = new_row >= 0 && new_row < nk && tid < 32;
+    const int nh = tid >> 4, nj = (tid >> 1) & 7, nwhich = tid & 1;  // 2 halves x 8 chunks x {K, V}
+    uint4 new_chunk = make_uint4(0u, 0u, 0u, 0u);
+    if (has_new)
+        new_chunk = __ldcg(reinterpret_cast<const uint4*>((nwhich ? vc : kc) +
+                                                          ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + nh * 64 + nj * 8));
+    const int qh = tid >> 4, qj = tid & 15;  // Q: head, 16-byte chunk of 8 dims (G * 16 <= kThreads)
+    float4 qa = make_float4(0.f, 0.f, 0.f, 0.f), qb = qa;
+    if (tid < G * 16) {
+        const float4* src = reinterpret_cast<const float4*>(q + (size_t)(kvh * G + qh) * kDH + qj * 8);
+        qa = __ldcg(src);
+        qb = __ldcg(src + 1);
+    }
+    if (warp == 0) {  // allocates and (at exit) frees the tensor memory
         tmem_alloc(&tmem_slot, kTmemCols);
         tmem_relinquish();
     }
@@ -119,38 +147,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    cluster_arrive_relaxed();  // waited on before the first push into another CTA's inbox
     const uint32_t tmem = tmem_slot;
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bar_kv, (uint32_t)nbox * 4u * kBoxBytes);
-        for (int b = 0; b < nbox; ++b) {
-            const int y = kb + b * kBoxRows;
-            for (int c = 0; c < 2; ++c) {
-                const uint32_t dst = half_off(p.rows, b >> 2, c) + (uint32_t)(b & 3) * kBoxBytes;
-                tma_load_3d(sK + dst, tmK, &bar_kv, c * 64, y, kvh);
-                tma_load_3d(sV + dst, tmV, &bar_kv, c * 64, y, kvh);
-            }
-        }
-    }
-    pdl_wait();
-    pdl_trigger();
-
     // Q (post-RoPE, fp32) -> bf16 rows [0, G) of the swizzled K-major tile
-    for (int i = tid; i < G * 16; i += kThreads) {
-        const int hh = i >> 4, j = i & 15;  // head, 16-byte chunk of 8 dims
-        const float4* src = reinterpret_cast<const float4*>(q + (size_t)(kvh * G + hh) * kDH + j * 8);
-        const float4 a = __ldcg(src), b = __ldcg(src + 1);
-        *reinterpret_cast<uint4*>(sQ + (j >> 3) * (16 * 128) + sw128_off(hh, j & 7)) =
-            make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w), pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
-    }
+    if (tid < G * 16)
+        *reinterpret_cast<uint4*>(sQ + (qj >> 3) * (16 * 128) + sw128_off(qh, qj & 7)) =
+            make_uint4(pack_bf16x2(qa.x, qa.y), pack_bf16x2(qa.z, qa.w), pack_bf16x2(qb.x, qb.y),
+                       pack_bf16x2(qb.z, qb.w));
     if (!mbar_wait(&bar_kv, 0)) s_ok = 0;
     // the new token's K and V rows over their (stale) slots; V rows past the range -> 0 so that
     // zero probabilities never meet non-finite values
-    if (new_row >= 0 && new_row < nk && tid < 32) {
-        const int half = tid >> 4, j = (tid >> 1) & 7, which = tid & 1;  // 2 halves x 8 chunks x {K, V}
-        const bf16* src = (which ? vc : kc) + ((size_t)kvh * p.max_ctx + (ctx - 1)) * kDH + half * 64 + j * 8;
-        uint8_t* dst = (which ? sV : sK) + half_off(p.rows, new_row >> 7, half) + sw128_off(new_row & 127, j);
-        *reinterpret_cast<uint4*>(dst) = __ldcg(reinterpret_cast<const uint4*>(src));
-    }
+    if (has_new)
+        *reinterpret_cast<uint4*>((nwhich ? sV : sK) + half_off(p.rows, new_row >> 7, nh) +
+                                  sw128_off(new_row & 127, nj)) = new_chunk;
     const int nt = (nk + 127) >> 7;
     const int zero_end = min(p.rows, (nk + 31) & ~31);  // rows the O MMA may read
     for (int i = nk * 16 + tid; i < zero_end * 16; i += kThreads) {  // (row, half, chunk) triples
@@ -257,6 +266,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         umma_commit(&bar_mma);
     }
+    // Push this CTA's partial state into the inbox of the rank that merges each element slice
+    // (every rank gets the per-head max and sum; those are complete since the barrier before
+    // the O MMA, so they go out while it runs), then one cluster barrier (release / acquire)
+    // makes every inbox complete; nothing reads another CTA's shared memory after it, so no
+    // second barrier is needed before exit.
+    cluster_wait();
+    for (int i = tid; i < p.cs * G; i += kThreads) {
+        const int q = i / G, hh = i % G;
+        float mv = -INFINITY, lv = 0.f;
+        if (run) {
+            mv = fmaxf(fmaxf(red_m[0][hh], red_m[1][hh]), fmaxf(red_m[2][hh], red_m[3][hh]));
+            lv = red_l[0][hh] + red_l[1][hh] + red_l[2][hh] + red_l[3][hh];
+        }
+        st_dsmem_f32(&rx_m[rank][hh], (uint32_t)q, mv);
+        st_dsmem_f32(&rx_l[rank][hh], (uint32_t)q, lv);
+    }
+    const int per_cta = G * kDH / p.cs;
     if (run) {
         if (!mbar_wait(&bar_mma, 1)) s_ok = 0;
         tc_fence_after();
@@ -264,39 +290,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + kOCol, r);
         const int d = warp * 32 + lane;
 #pragma unroll
-        for (int hh = 0; hh < G; ++hh) c_o[hh * kDH + d] = __uint_as_float(r[hh]);
-        if (tid < G) {
-            c_m[tid] = m_loc[tid];
-            c_l[tid] = red_l[0][tid] + red_l[1][tid] + red_l[2][tid] + red_l[3][tid];
+        for (int hh = 0; hh < G; ++hh) {
+            const int e = hh * kDH + d;
+            st_dsmem_f32(&rx_o[rank][e % per_cta], (uint32_t)(e / per_cta), __uint_as_float(r[hh]));
         }
     } else {
-        for (int i = tid; i < G * kDH; i += kThreads) c_o[i] = 0.f;
-        if (tid < G) {
-            c_m[tid] = -INFINITY;
-            c_l[tid] = 0.f;
-        }
+        for (int e = tid; e < G * kDH; e += kThreads)
+            st_dsmem_f32(&rx_o[rank][e % per_cta], (uint32_t)(e / per_cta), 0.f);
     }
     tc_fence_before();
-    __syncthreads();
+    cluster_sync_all();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
     if (!s_ok && tid == 0) set_status(p.status, kDevTimeout);
-    // push this CTA's partial state to the rank that merges each element slice, then one
-    // cluster barrier (release / acquire) makes every inbox complete; nothing reads another
-    // CTA's shared memory after it, so no second barrier is needed before exit
-    const int per_cta = G * kDH / p.cs;
-    for (int i = tid; i < p.cs * per_cta; i += kThreads) {
-        const int q = i / per_cta, k = i % per_cta;
-        st_dsmem_f32(&rx_o[rank][k], (uint32_t)q, c_o[q * per_cta + k]);
-    }
-    for (int i = tid; i < p.cs * G; i += kThreads) {
-        const int q = i / G, hh = i % G;
-        st_dsmem_f32(&rx_m[rank][hh], (uint32_t)q, c_m[hh]);
-        st_dsmem_f32(&rx_l[rank][hh], (uint32_t)q, c_l[hh]);
-    }
-    cluster_sync_all();
     if (tid < per_cta) {
         const int e = rank * per_cta + tid;
         const int hh = e / kDH;
