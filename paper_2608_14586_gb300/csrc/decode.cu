@@ -21,6 +21,7 @@
 // predate the step before the wait, so the copy overlaps the QKV kernel), scores it for all
 // query heads of the GQA group with an online softmax, and the cluster merges the partial
 // (max, sum, output) states through distributed shared memory in fixed rank order.
+#include <algorithm>
 #include <cstring>
 
 #include "common.cuh"
@@ -58,6 +59,7 @@ constexpr int kGemvThreads = 256;
 constexpr int kGemvWarps = kGemvThreads / 32;
 constexpr int kGemvSegBytes = 4096;  // bytes of each row per ring slot
 constexpr int kGemvMaxStages = 3;
+constexpr size_t kGemvSmemBudget = 226 * 1024;  // dynamic shared memory of one CTA (of 227 KB)
 
 VLA_DEV float dot8(uint4 w, uint4 x) {
     float a = bf16_lo(w.x) * bf16_lo(x.x);
@@ -506,8 +508,13 @@ template <int MODE, int NB>
 cudaError_t launch_gemv_nb(const GemvParams& p_in, int num_sms, cudaStream_t s, bool pdl) {
     GemvParams p = p_in;
     if (p.K % 256 != 0 || p.units <= 0) return cudaErrorInvalidValue;
-    p.stages = NB == 1 ? 3 : 2;  // ring slots per warp within the shared memory of one CTA per SM
-    const size_t smem = (size_t)NB * p.K * 2 + (size_t)kGemvWarps * p.stages * 2 * kGemvSegBytes;
+    // as many ring slots per warp (up to three) as the shared memory of one CTA per SM holds
+    // beside the NB input vectors
+    const size_t xbytes = (size_t)NB * p.K * 2;
+    const size_t slot_bytes = (size_t)kGemvWarps * 2 * kGemvSegBytes;
+    if (xbytes + slot_bytes > kGemvSmemBudget) return cudaErrorInvalidValue;
+    p.stages = (int)std::min<size_t>(kGemvMaxStages, (kGemvSmemBudget - xbytes) / slot_bytes);
+    const size_t smem = xbytes + (size_t)p.stages * slot_bytes;
     auto kern = gemv_kernel<MODE, NB>;
     static size_t attr = 0;
     if (smem > attr) {
