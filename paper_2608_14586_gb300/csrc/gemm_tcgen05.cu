@@ -292,6 +292,21 @@ VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     }
 }
 
+// 32 lanes x 32 fp32 columns at each of two TMEM addresses, one wait for both loads
+VLA_DEV void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t (&a)[32], uint32_t (&b)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%64];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%65];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n"
+        : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]), "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]), "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]), "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+        : "r"(ta), "r"(tb)
+        : "memory");
+}
+
+// SiLU(g) * u with g, u the gate and up accumulators scaled by 1/rms. The division is the
+// fast reciprocal form (__fdividef: within 2 ulp of fp32, far below the bf16 rounding of the
+// stored value; for g below about -87 the denominator overflows and the product is 0, the
+// function's limit).
 template <int BN>
 VLA_DEV void epi_swiglu(uint32_t taddr, int row, int n0, const EpiParams& ep) {
     constexpr int HALF = BN / 2;
@@ -301,15 +316,14 @@ VLA_DEV void epi_swiglu(uint32_t taddr, int row, int n0, const EpiParams& ep) {
 #pragma unroll 1
     for (int c = 0; c < HALF; c += 32) {
         uint32_t rg[32], ru[32];
-        tmem_ld32(taddr + c, rg);
-        tmem_ld32(taddr + HALF + c, ru);
+        tmem_ld32x2(taddr + c, taddr + HALF + c, rg, ru);
         if (!row_ok) continue;
         float v[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
             const float g = f32(rg[i]) * s;
             const float u = f32(ru[i]) * s;
-            v[i] = g / (1.0f + __expf(-g)) * u;
+            v[i] = __fdividef(g, 1.0f + __expf(-g)) * u;
         }
         store_bf16x32(ep.out + (size_t)row * ep.ld_out + f0 + c, v);
     }
