@@ -87,6 +87,39 @@ def test_7b_block_1024_tokens(vla_lib):
         m.close()
 
 
+def test_7b_block_512_tokens_every_row_and_repeatable(vla_lib):
+    """One 7B block at 512 tokens (the gate/up GEMM's 344 tiles take two rounds and 40 tiles
+    of a third on 152 SMs), every output row against the oracle, and a second run must give
+    the same bits."""
+    import torch
+    vla = vla_lib
+    s = synth.B7
+    M = 512
+    m = Model(s, 1, 5, M)
+    try:
+        xb = synth.hidden_states(M, s.hidden, 5)
+        x = to_dev(xb)
+        cache = oracle.KVCache([0], s.n_kv_heads, s.head_dim, M)
+        ref = oracle.prefix_forward(oracle.bf16_to_f64(xb), m.weights64(), 0, 1, cache, s)
+        kv = vla.vla_kv_create(m.handle, 0, 1, M)
+        y = torch.empty_like(x)
+        outs = []
+        for _ in range(2):
+            vla.vla_kv_set_length(kv, 0)
+            vla.vla_prefix_prefill(m.handle, x, M, 0, 1, kv, y)
+            sync()
+            assert vla.vla_last_async_error(m.handle) == 0
+            outs.append(y.clone())
+        assert torch.equal(outs[0].view(torch.int16), outs[1].view(torch.int16))
+        got = from_dev(outs[0])
+        assert rel_l2(got, ref) < REL_L2_BLOCK
+        row_err = np.linalg.norm(got - ref, axis=1) / np.linalg.norm(ref, axis=1)
+        assert row_err.max() < 2 * REL_L2_BLOCK
+        vla.vla_kv_destroy(kv)
+    finally:
+        m.close()
+
+
 def test_prefill_continues_context_and_random_gains(vla_lib):
     """Two prefills on one cache (positions 0..99 then 100..136) with non-unit RMSNorm gains."""
     import torch
