@@ -3,14 +3,18 @@
 // One thread-block cluster of `cs` CTAs per (sequence, KV head g); CTA rank r owns the contiguous key range
 // [r*ceil(ctx/cs), ...) of the context (the attention stage of a block, Sec. IV-B, at one query
 // position, split over keys). Per CTA, for the G query heads of the GQA group:
-//   1. TMA copies the range's K and V rows (32-row boxes, 128-byte swizzle) into shared memory
-//      sized to the range (two CTAs fit on an SM, so all Hkv clusters of 16 are co-resident).
-//      Rows that predate this step are requested before griddepcontrol.wait, so the copy
-//      overlaps the QKV kernel; the new token's row is written over its slot afterwards.
-//   2. S^T = K Q^T on tcgen05 (M = 128 keys per tile, N = 16 >= G heads, K = d_h), fp32 in TMEM.
+//   1. First thing, the lanes of warp 0 issue TMA copies of the range's K and V rows that
+//      predate this step (32-row boxes, 128-byte swizzle) into shared memory sized to the
+//      range; after griddepcontrol.wait, Q and the new token's K and V rows are read while
+//      tensor memory is allocated, then written into shared memory (the new rows over their
+//      slots).
+//   2. S^T = K Q^T on tcgen05 per 128-key tile (M = 128 keys, N = 16 >= G heads, K = d_h),
+//      fp32 in TMEM; lane 0 of warp t issues tile t, so the tiles' MMAs go out in parallel.
 //   3. One thread per key row reads its G scores, the CTA takes the per-head max and sum of
 //      exp2(s * log2(e)/sqrt(d_h) - max), and writes P^T (bf16, 128-byte-swizzled K-major).
-//   4. O^T = V^T P^T on tcgen05 (M = d_h, N = 16, K = keys; V^T read MN-major in place).
+//   4. O^T partial of tile t = V_t^T P_t^T on tcgen05 (M = d_h, N = 16, K = the tile's keys;
+//      V^T read MN-major in place), again one issuing thread per tile; the partials are added
+//      in tile order when they are read.
 //   5. Each CTA stores its (max, sum, unnormalised O) through distributed shared memory into
 //      the inbox of the rank that merges each element slice; after one cluster barrier CTA r
 //      merges output elements [r*G*d_h/cs, (r+1)*G*d_h/cs) from its inbox in fixed rank order
@@ -32,8 +36,8 @@ constexpr int kMaxRows = 384;                       // keys per CTA (3 tiles)
 constexpr uint32_t kQBytes = 2u * 16u * 128u;       // [16 rows][128] as two halves of 64
 constexpr uint32_t kPTileBytes = 2u * 16u * 128u;   // [16 heads][128 keys] as two halves of 64
 constexpr uint32_t kBoxBytes = kBoxRows * 128u;     // one [32 rows][64] box
-constexpr uint32_t kTmemCols = 64;                  // S^T tiles at [16t, 16t+16), O^T at [48, 64)
-constexpr uint32_t kOCol = 48;
+constexpr uint32_t kTmemCols = 128;  // S^T of tile t at [16t, 16t+16), its O^T partial at [64+16t, ...)
+constexpr uint32_t kOCol = 64;
 constexpr int kMaxCs = 16;
 
 // byte offset of (row, 16-byte chunk j) inside a 128-byte-swizzled tile of 128-byte rows
@@ -68,7 +72,7 @@ template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_decode_tc_kernel(const __grid_constant__ DecKVMaps maps, const __grid_constant__ AttnDecTcParams p) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ uint64_t bar_kv, bar_mma;
+    __shared__ uint64_t bar_kv, bar_s[3], bar_o[3];  // K/V landed; per 128-key tile: S^T, O^T done
     __shared__ uint32_t tmem_slot;
     __shared__ float red_m[4][G], red_l[4][G];
     // merge inbox: from each rank of the cluster, its (max, sum) per head and its unnormalised
@@ -104,7 +108,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             mbar_init(&bar_kv, 1);
-            mbar_init(&bar_mma, 1);
+            for (int t = 0; t < 3; ++t) {
+                mbar_init(&bar_s[t], 1);
+                mbar_init(&bar_o[t], 1);
+            }
             fence_barrier_init();
             s_ok = 1;
             mbar_arrive_expect_tx(&bar_kv, (uint32_t)nbox * 4u * kBoxBytes);
@@ -171,27 +178,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     const bool run = s_ok && nk > 0;  // CTA-uniform
 
-    // S^T = K Q^T, one 128-key tile at a time, into TMEM columns [16t, 16t + 16)
-    if (run && tid == 0) {
+    // S^T = K Q^T of 128-key tile t into TMEM columns [16t, 16t + 16), issued by lane 0 of
+    // warp t (the tiles' MMAs go out in parallel)
+    if (run && lane == 0 && warp < nt) {
+        const int t = warp;
         tc_fence_after();
         constexpr uint32_t idesc = idesc_bf16_f32(128, 16);
-        for (int t = 0; t < nt; ++t) {
-            const uint32_t qt = smem_u32(sQ);
+        const uint32_t qt = smem_u32(sQ);
 #pragma unroll
-            for (int kk = 0; kk < kDH / 16; ++kk) {
-                const uint64_t ad = sw128_kmajor_desc(smem_u32(sK + half_off(p.rows, t, kk >> 2))) + 2 * (kk & 3);
-                const uint64_t bd = sw128_kmajor_desc(qt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
-                umma_bf16_ss(tmem + t * 16, ad, bd, idesc, kk > 0 ? 1u : 0u);
-            }
+        for (int kk = 0; kk < kDH / 16; ++kk) {
+            const uint64_t ad = sw128_kmajor_desc(smem_u32(sK + half_off(p.rows, t, kk >> 2))) + 2 * (kk & 3);
+            const uint64_t bd = sw128_kmajor_desc(qt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
+            umma_bf16_ss(tmem + t * 16, ad, bd, idesc, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&bar_mma);
+        umma_commit(&bar_s[t]);
     }
     float s[3][G];
     float m_loc[G], l_loc[G];
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) m_loc[hh] = -INFINITY, l_loc[hh] = 0.f;
     if (run) {
-        if (!mbar_wait(&bar_mma, 0)) s_ok = 0;
+        for (int t = 0; t < nt; ++t)
+            if (!mbar_wait(&bar_s[t], 0)) s_ok = 0;
         tc_fence_after();
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll
@@ -249,22 +257,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
     }
     __syncthreads();
-    // O^T = V^T P^T into TMEM columns [48, 64): A = V tile read MN-major (M = d_h), B = P^T
-    if (run && tid == 0) {
+    // O^T partial of tile t = V_t^T P_t^T into TMEM columns [64 + 16t, ...), issued by lane 0 of
+    // warp t: A = V tile read MN-major (M = d_h), B = P^T; the partials are added at readout
+    if (run && lane == 0 && warp < nt) {
+        const int t = warp;
         tc_fence_after();
         constexpr uint32_t idesc = idesc_bf16_f32(128, 16) | (1u << 15);
-        for (int t = 0; t < nt; ++t) {
-            const uint32_t vt = smem_u32(sV + half_off(p.rows, t, 0));
-            const uint32_t vstride = half_off(p.rows, t, 1) - half_off(p.rows, t, 0);
-            const uint32_t pt = smem_u32(sP + t * kPTileBytes);
-            const int steps = (min(128, nk - 128 * t) + 15) >> 4;  // 16-key steps holding keys
-            for (int kk = 0; kk < steps; ++kk) {
-                const uint64_t ad = sw128_mnmajor_desc(vt + kk * 16 * 128, vstride);
-                const uint64_t bd = sw128_kmajor_desc(pt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
-                umma_bf16_ss(tmem + kOCol, ad, bd, idesc, (t > 0 || kk > 0) ? 1u : 0u);
-            }
+        const uint32_t vt = smem_u32(sV + half_off(p.rows, t, 0));
+        const uint32_t vstride = half_off(p.rows, t, 1) - half_off(p.rows, t, 0);
+        const uint32_t pt = smem_u32(sP + t * kPTileBytes);
+        const int steps = (min(128, nk - 128 * t) + 15) >> 4;  // 16-key steps holding keys
+        for (int kk = 0; kk < steps; ++kk) {
+            const uint64_t ad = sw128_mnmajor_desc(vt + kk * 16 * 128, vstride);
+            const uint64_t bd = sw128_kmajor_desc(pt + (kk >> 2) * (16 * 128)) + 2 * (kk & 3);
+            umma_bf16_ss(tmem + kOCol + t * 16, ad, bd, idesc, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&bar_mma);
+        umma_commit(&bar_o[t]);
     }
     // Push this CTA's partial state into the inbox of the rank that merges each element slice
     // (every rank gets the per-head max and sum; those are complete since the barrier before
@@ -284,15 +292,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     const int per_cta = G * kDH / p.cs;
     if (run) {
-        if (!mbar_wait(&bar_mma, 1)) s_ok = 0;
+        for (int t = 0; t < nt; ++t)
+            if (!mbar_wait(&bar_o[t], 0)) s_ok = 0;
         tc_fence_after();
-        uint32_t r[16];
-        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + kOCol, r);
+        float o[G];
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) o[hh] = 0.f;
+#pragma unroll
+        for (int t = 0; t < 3; ++t) {  // the tiles' partials, added in tile order
+            if (t < nt) {
+                uint32_t r[16];
+                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + kOCol + t * 16, r);
+#pragma unroll
+                for (int hh = 0; hh < G; ++hh) o[hh] += __uint_as_float(r[hh]);
+            }
+        }
         const int d = warp * 32 + lane;
 #pragma unroll
         for (int hh = 0; hh < G; ++hh) {
             const int e = hh * kDH + d;
-            st_dsmem_f32(&rx_o[rank][e % per_cta], (uint32_t)(e / per_cta), __uint_as_float(r[hh]));
+            st_dsmem_f32(&rx_o[rank][e % per_cta], (uint32_t)(e / per_cta), o[hh]);
         }
     } else {
         for (int e = tid; e < G * kDH; e += kThreads)
