@@ -244,54 +244,6 @@ VLA_DEV void store_bf16x16(bf16* dst, const float* v) {
     }
 }
 
-// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
-// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
-// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
-// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order.
-template <int BN>
-VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
-    const bool row_ok = row < ep.M;
-    const float s = row_ok ? row_rinv(ep, row) : 0.f;
-    const int pos = ep.pos0 + row;
-    const int dh = ep.head_dim;
-    const int half = dh >> 1;
-    const float2* rope = ep.rope + (size_t)(row_ok ? pos : 0) * half;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-        uint32_t r[32];
-        tmem_ld32(taddr + c, r);
-        const int col = n0 + c;
-        if (!row_ok || col >= ep.N) continue;
-        if (col >= ep.q_cols + ep.kv_cols) {
-            const int n = col - ep.q_cols - ep.kv_cols;
-            const int g = n / dh, d = n % dh;
-            float v[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = f32(r[i]) * s;
-            store_bf16x32(ep.vcache + ((size_t)g * ep.max_ctx + pos) * dh + d, v);
-            continue;
-        }
-        const bool is_q = col < ep.q_cols;
-        const int n = is_q ? col : col - ep.q_cols;
-        const int head = n / dh, i0 = (n % dh) >> 1;
-        float va[16], vb[16];
-#pragma unroll
-        for (int i = 0; i < 16; i += 2) {  // 16-byte loads: two (cos, sin) pairs each
-            const float4 cs = __ldg(reinterpret_cast<const float4*>(rope + i0 + i));
-            const float a0 = f32(r[2 * i]) * s, b0 = f32(r[2 * i + 1]) * s;
-            const float a1 = f32(r[2 * i + 2]) * s, b1 = f32(r[2 * i + 3]) * s;
-            va[i] = a0 * cs.x - b0 * cs.y;
-            vb[i] = b0 * cs.x + a0 * cs.y;
-            va[i + 1] = a1 * cs.z - b1 * cs.w;
-            vb[i + 1] = b1 * cs.z + a1 * cs.w;
-        }
-        bf16* dst = is_q ? ep.out + (size_t)row * ep.ld_out + (size_t)head * dh
-                         : ep.kcache + ((size_t)head * ep.max_ctx + pos) * dh;
-        store_bf16x16(dst + i0, va);
-        store_bf16x16(dst + i0 + half, vb);
-    }
-}
-
 // 32 lanes x 32 fp32 columns at each of two TMEM addresses, one wait for both loads
 VLA_DEV void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t (&a)[32], uint32_t (&b)[32]) {
     asm volatile(
@@ -301,6 +253,93 @@ VLA_DEV void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t (&a)[32], uint32_t (
         : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]), "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]), "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]), "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
         : "r"(ta), "r"(tb)
         : "memory");
+}
+
+// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
+// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
+// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
+// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order.
+// One 32-column chunk at output column `col` of the QKV epilogue; cs: the chunk's 16 (cos, sin)
+// pairs, two per float4 (q and k chunks only).
+VLA_DEV void qkv_chunk(const uint32_t (&r)[32], int col, const float4 (&cs)[8], float s, int row, int pos,
+                       const EpiParams& ep) {
+    const int dh = ep.head_dim;
+    if (col >= ep.q_cols + ep.kv_cols) {
+        const int n = col - ep.q_cols - ep.kv_cols;
+        const int g = n / dh, d = n % dh;
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]) * s;
+        store_bf16x32(ep.vcache + ((size_t)g * ep.max_ctx + pos) * dh + d, v);
+        return;
+    }
+    const bool is_q = col < ep.q_cols;
+    const int n = is_q ? col : col - ep.q_cols;
+    const int head = n / dh, i0 = (n % dh) >> 1;
+    float va[16], vb[16];
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+        const float4 c4 = cs[i >> 1];
+        const float a0 = f32(r[2 * i]) * s, b0 = f32(r[2 * i + 1]) * s;
+        const float a1 = f32(r[2 * i + 2]) * s, b1 = f32(r[2 * i + 3]) * s;
+        va[i] = a0 * c4.x - b0 * c4.y;
+        vb[i] = b0 * c4.x + a0 * c4.y;
+        va[i + 1] = a1 * c4.z - b1 * c4.w;
+        vb[i + 1] = b1 * c4.z + a1 * c4.w;
+    }
+    bf16* dst = is_q ? ep.out + (size_t)row * ep.ld_out + (size_t)head * dh
+                     : ep.kcache + ((size_t)head * ep.max_ctx + pos) * dh;
+    store_bf16x16(dst + i0, va);
+    store_bf16x16(dst + i0 + (dh >> 1), vb);
+}
+
+// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
+// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
+// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
+// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order. With 256-column tiles and
+// d_h = 128 the chunks c and c + 4 are the same dims of two heads: they are read from tensor
+// memory with one wait and share one load of the row's (cos, sin) pairs.
+template <int BN>
+VLA_DEV void epi_qkv(uint32_t taddr, int row, int n0, const EpiParams& ep) {
+    const bool row_ok = row < ep.M;
+    const float s = row_ok ? row_rinv(ep, row) : 0.f;
+    const int pos = ep.pos0 + row;
+    const int dh = ep.head_dim;
+    const int half = dh >> 1;
+    const int rope_cols = ep.q_cols + ep.kv_cols;  // columns [0, rope_cols) are rotated
+    const float2* rope = ep.rope + (size_t)(row_ok ? pos : 0) * half;
+    if (BN == 256 && dh == 128) {
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+            const int col = n0 + 32 * c;  // and col + 128: the same dims of the next head
+            const int i0 = (col % dh) >> 1;
+            float4 cs[8];
+            if (row_ok && (col < rope_cols || col + 128 < rope_cols)) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) cs[i] = __ldg(reinterpret_cast<const float4*>(rope + i0 + 2 * i));
+            }
+            uint32_t ra[32], rb[32];
+            tmem_ld32x2(taddr + 32 * c, taddr + 32 * c + 128, ra, rb);
+            if (!row_ok) continue;
+            if (col < ep.N) qkv_chunk(ra, col, cs, s, row, pos, ep);
+            if (col + 128 < ep.N) qkv_chunk(rb, col + 128, cs, s, row, pos, ep);
+        }
+        return;
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+        const int col = n0 + c;
+        float4 cs[8];
+        if (row_ok && col < rope_cols) {
+            const int i0 = (col % dh) >> 1;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) cs[i] = __ldg(reinterpret_cast<const float4*>(rope + i0 + 2 * i));
+        }
+        uint32_t r[32];
+        tmem_ld32(taddr + c, r);
+        if (!row_ok || col >= ep.N) continue;
+        qkv_chunk(r, col, cs, s, row, pos, ep);
+    }
 }
 
 // SiLU(g) * u with g, u the gate and up accumulators scaled by 1/rms. The division is the
