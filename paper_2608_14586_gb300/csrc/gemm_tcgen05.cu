@@ -67,6 +67,21 @@ VLA_DEV void store_bf16x32(bf16* dst, const float (&v)[32]) {
 // Epilogues. Each thread owns one output row (TMEM lane); all 32 lanes of a warp execute
 // every tcgen05.ld; stores are masked per row / column.
 // ---------------------------------------------------------------------------------------
+// 32 lanes x 32 fp32 columns at each of two TMEM addresses, one wait for both loads
+VLA_DEV void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t (&a)[32], uint32_t (&b)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%64];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%65];\n\t"
+        "tcgen05.wait::ld.sync.aligned;\n"
+        : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]), "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]), "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]), "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+        : "r"(ta), "r"(tb)
+        : "memory");
+}
+
+// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
+// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
+// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
+// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order.
 // 1/rms of an input row from its 32-column partial sums of squares, added in group order
 VLA_DEV float row_rinv(const EpiParams& ep, int row) {
     const float* ps = ep.ss_in + (size_t)row * ep.ss_groups;
@@ -156,77 +171,88 @@ VLA_DEV void epi_plain_resid(uint32_t taddr, int row, int n0, const EpiParams& e
 // 32 rows is packed into a 32 x 32 bf16 box in shared memory (64-byte swizzle, so the 16-byte
 // writes of the 32 lanes spread over all banks) and one lane stores the box with
 // cp.async.bulk.tensor; the box rows past M and columns past N are clipped by the tensor map.
-// Two boxes per warp alternate, the older store's read of its box waited for before reuse.
-// Needs N a multiple of 32 and no host copy (out_host). Row statistics as epi_plain_resid.
+// Chunks go in pairs: one tensor-memory wait for both, both boxes of the warp filled, one
+// proxy fence, two stores in one bulk group (the previous pair's group has read its boxes
+// before they are refilled). Needs N a multiple of 32, an even chunk count and no host copy
+// (out_host). Row statistics as epi_plain_resid.
 template <int BN>
 VLA_DEV void epi_resid_tma(uint32_t taddr, int row, int row0, int n0, const EpiParams& ep, const CUtensorMap* tm_out,
                            uint8_t* stage, uint32_t& nstore, int lane) {
     constexpr int NC = BN / 32;
+    static_assert(NC % 2 == 0, "chunk pairs");
     const bool row_ok = row < ep.M;
     const bool has_res = row_ok && ep.resid != nullptr;
     const uint4* rrow = has_res ? reinterpret_cast<const uint4*>(ep.resid + (size_t)row * ep.ld_resid + n0) : nullptr;
-    // the residual chunks are requested two ahead of their use, so their latency overlaps the
-    // tensor-memory reads and the stores of the chunks before
-    uint4 res[3][4];
+    // the residual chunks are requested one pair ahead of their use, so their latency overlaps
+    // the tensor-memory reads and the stores of the pair before
+    uint4 res[4][4];
     auto fetch = [&](int c) {
         if (has_res && n0 + 32 * c < ep.N) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) res[c % 3][i] = rrow[4 * c + i];
+            for (int i = 0; i < 4; ++i) res[c % 4][i] = rrow[4 * c + i];
         }
     };
     fetch(0);
-    if (NC > 1) fetch(1);
+    fetch(1);
     float ss = 0.f;
 #pragma unroll
-    for (int c = 0; c < NC; ++c) {
-        if (c + 2 < NC) fetch(c + 2);
-        uint32_t r[32];
-        tmem_ld32(taddr + 32 * c, r);
-        const int col = n0 + 32 * c;
-        if (col >= ep.N) continue;  // uniform over the warp
-        float v[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = f32(r[i]);
-        if (has_res) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint4 q = res[c % 3][i];
-                v[i * 8 + 0] += bf16_lo(q.x);
-                v[i * 8 + 1] += bf16_hi(q.x);
-                v[i * 8 + 2] += bf16_lo(q.y);
-                v[i * 8 + 3] += bf16_hi(q.y);
-                v[i * 8 + 4] += bf16_lo(q.z);
-                v[i * 8 + 5] += bf16_hi(q.z);
-                v[i * 8 + 6] += bf16_lo(q.w);
-                v[i * 8 + 7] += bf16_hi(q.w);
-            }
+    for (int c = 0; c < NC; c += 2) {
+        if (c + 2 < NC) {
+            fetch(c + 2);
+            fetch(c + 3);
         }
-        if (ep.ss_out && row_ok) {  // the group's sum of squares of the stored values, a chain from zero
-            float g = 0.f;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const float rr = __bfloat162float(__float2bfloat16_rn(v[i]));
-                g = fmaf(rr, rr, g);
-            }
-            if (ep.ss_width == 32) ep.ss_out[(size_t)row * ep.ss_groups + (col >> 5)] = g;
-            else ss += g;
-        }
-        uint8_t* box = stage + (nstore & 1u) * 2048u;
-        if (lane == 0) bulk_wait_group_read<1>();  // the store that last used this box has read it
+        uint32_t r2[2][32];
+        tmem_ld32x2(taddr + 32 * c, taddr + 32 * (c + 1), r2[0], r2[1]);
+        if (n0 + 32 * c >= ep.N) continue;  // uniform over the warp (then so is the second chunk)
+        if (lane == 0) bulk_wait_group_read<0>();  // the previous pair's stores have read both boxes
         __syncwarp();
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const uint4 o = make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
-            *reinterpret_cast<uint4*>(box + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = o;
+        for (int j = 0; j < 2; ++j) {
+            const int col = n0 + 32 * (c + j);
+            if (col >= ep.N) continue;
+            float v[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = f32(r2[j][i]);
+            if (has_res) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint4 q = res[(c + j) % 4][i];
+                    v[i * 8 + 0] += bf16_lo(q.x);
+                    v[i * 8 + 1] += bf16_hi(q.x);
+                    v[i * 8 + 2] += bf16_lo(q.y);
+                    v[i * 8 + 3] += bf16_hi(q.y);
+                    v[i * 8 + 4] += bf16_lo(q.z);
+                    v[i * 8 + 5] += bf16_hi(q.z);
+                    v[i * 8 + 6] += bf16_lo(q.w);
+                    v[i * 8 + 7] += bf16_hi(q.w);
+                }
+            }
+            if (ep.ss_out && row_ok) {  // the group's sum of squares of the stored values, a chain from zero
+                float g = 0.f;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float rr = __bfloat162float(__float2bfloat16_rn(v[i]));
+                    g = fmaf(rr, rr, g);
+                }
+                if (ep.ss_width == 32) ep.ss_out[(size_t)row * ep.ss_groups + (col >> 5)] = g;
+                else ss += g;
+            }
+            uint8_t* box = stage + (uint32_t)j * 2048u;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 o = make_uint4(pack_bf16x2(v[8 * q + 0], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                           pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+                *reinterpret_cast<uint4*>(box + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = o;
+            }
         }
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-            tma_store_2d(tm_out, box, col, row0);
+            tma_store_2d(tm_out, stage, n0 + 32 * c, row0);
+            if (n0 + 32 * (c + 1) < ep.N) tma_store_2d(tm_out, stage + 2048u, n0 + 32 * (c + 1), row0);
             bulk_commit_group();
         }
-        ++nstore;
+        nstore += 2;
     }
     if (ep.ss_out && ep.ss_width == 256 && row_ok && n0 < ep.N) ep.ss_out[(size_t)row * ep.ss_groups + n0 / 256] = ss;
 }
@@ -244,21 +270,6 @@ VLA_DEV void store_bf16x16(bf16* dst, const float* v) {
     }
 }
 
-// 32 lanes x 32 fp32 columns at each of two TMEM addresses, one wait for both loads
-VLA_DEV void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t (&a)[32], uint32_t (&b)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%64];\n\t"
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%65];\n\t"
-        "tcgen05.wait::ld.sync.aligned;\n"
-        : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]), "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]), "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]), "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]), "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]), "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]), "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]), "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
-        : "r"(ta), "r"(tb)
-        : "memory");
-}
-
-// Per 32-column chunk (each inside one of the q, k, v regions, whose widths are multiples of
-// 32): q and k columns hold rotation pairs side by side (columns 2j, 2j+1 of a head = dims j,
-// j + dh/2), so a chunk is 16 whole pairs; their rotated values go to dims [i0, i0+16) and
-// [i0 + dh/2, i0 + dh/2 + 16). Value columns are in natural order.
 // One 32-column chunk at output column `col` of the QKV epilogue; cs: the chunk's 16 (cos, sin)
 // pairs, two per float4 (q and k chunks only).
 VLA_DEV void qkv_chunk(const uint32_t (&r)[32], int col, const float4 (&cs)[8], float s, int row, int pos,
@@ -572,10 +583,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else if constexpr (EPI == kEpiSwiGLU) {
                 epi_swiglu<BN>(taddr, row, n0, ep);
             } else {
-                if (C::OUT_BYTES && ep.tma_out)
-                    epi_resid_tma<BN>(taddr, row, m0 + quarter * 32, n0, ep, &tmOut, stage_out, nstore, lane);
-                else
+                if constexpr (C::OUT_BYTES != 0) {  // 256-column tiles: a staging box pair per warp
+                    if (ep.tma_out)
+                        epi_resid_tma<BN>(taddr, row, m0 + quarter * 32, n0, ep, &tmOut, stage_out, nstore, lane);
+                    else
+                        epi_plain_resid<BN>(taddr, row, n0, ep);
+                } else {
                     epi_plain_resid<BN>(taddr, row, n0, ep);
+                }
             }
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
