@@ -205,3 +205,29 @@ def test_prefill_to_host_fused_boundary_store(vla_lib, shape_name, L, M):
         vla.vla_kv_destroy(kv)
     finally:
         m.close()
+
+
+def test_frame_to_device_uploads_pinned_frames_and_rejects_pageable_ones(vla_lib):
+    """The frame's input hand-off: page-locked host bits arrive unchanged in the device buffer
+    (on the caller's stream, ordered with work recorded after it); a pageable source is
+    refused with NOT_PINNED and leaves the buffer alone; zero tokens copy nothing."""
+    import torch
+    lib = vla_lib.load()
+    M, D = 300, 256
+    bits = synth.hidden_states(M, D, 3)
+    host = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).pin_memory()
+    dev = torch.zeros((M, D), dtype=torch.bfloat16, device="cuda")
+    s = torch.cuda.Stream()
+    vla_lib.vla_frame_to_device(host, M, D, dev, s)
+    done = torch.cuda.Event()
+    done.record(s)
+    done.synchronize()
+    np.testing.assert_array_equal(_bits(dev), np.asarray(bits).view(np.int16).reshape(M, D))
+    pageable = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+    dev2 = torch.zeros((M, D), dtype=torch.bfloat16, device="cuda")
+    assert lib.vla_frame_to_device(ctypes.c_void_p(pageable.data_ptr()), M, D, ctypes.c_void_p(dev2.data_ptr()),
+                                   None) == 5  # VLA_ERR_NOT_PINNED
+    assert lib.vla_frame_to_device(ctypes.c_void_p(host.data_ptr()), 0, D, ctypes.c_void_p(dev2.data_ptr()),
+                                   None) == 0
+    sync()
+    assert not dev2.view(torch.int16).any()
