@@ -61,15 +61,36 @@ constexpr int kGemvSegBytes = 4096;  // bytes of each row per ring slot
 constexpr int kGemvMaxStages = 3;
 constexpr size_t kGemvSmemBudget = 226 * 1024;  // dynamic shared memory of one CTA (of 227 KB)
 
+// a * b + c on the low (HI false) or high bf16 halves of two packed words, rounded once to
+// fp32 by the mixed-precision fma: a bf16 product is exact in fp32, so this is fmaf on the
+// widened values, without the widening instructions
+template <bool HI>
+VLA_DEV float fma_bf16(uint32_t a, uint32_t b, float c) {
+    float d;
+    if constexpr (HI)
+        asm("{\n\t.reg .b16 al, ah, bl, bh;\n\tmov.b32 {al, ah}, %1;\n\tmov.b32 {bl, bh}, %2;\n\t"
+            "fma.rn.f32.bf16 %0, ah, bh, %3;\n\t}"
+            : "=f"(d)
+            : "r"(a), "r"(b), "f"(c));
+    else
+        asm("{\n\t.reg .b16 al, ah, bl, bh;\n\tmov.b32 {al, ah}, %1;\n\tmov.b32 {bl, bh}, %2;\n\t"
+            "fma.rn.f32.bf16 %0, al, bl, %3;\n\t}"
+            : "=f"(d)
+            : "r"(a), "r"(b), "f"(c));
+    return d;
+}
+
+// sum of the eight products of two packed bf16 vectors, in order (the first product alone:
+// adding -0 keeps the sign of a zero product, as a plain multiply would)
 VLA_DEV float dot8(uint4 w, uint4 x) {
-    float a = bf16_lo(w.x) * bf16_lo(x.x);
-    a = fmaf(bf16_hi(w.x), bf16_hi(x.x), a);
-    a = fmaf(bf16_lo(w.y), bf16_lo(x.y), a);
-    a = fmaf(bf16_hi(w.y), bf16_hi(x.y), a);
-    a = fmaf(bf16_lo(w.z), bf16_lo(x.z), a);
-    a = fmaf(bf16_hi(w.z), bf16_hi(x.z), a);
-    a = fmaf(bf16_lo(w.w), bf16_lo(x.w), a);
-    a = fmaf(bf16_hi(w.w), bf16_hi(x.w), a);
+    float a = fma_bf16<false>(w.x, x.x, -0.0f);
+    a = fma_bf16<true>(w.x, x.x, a);
+    a = fma_bf16<false>(w.y, x.y, a);
+    a = fma_bf16<true>(w.y, x.y, a);
+    a = fma_bf16<false>(w.z, x.z, a);
+    a = fma_bf16<true>(w.z, x.z, a);
+    a = fma_bf16<false>(w.w, x.w, a);
+    a = fma_bf16<true>(w.w, x.w, a);
     return a;
 }
 
