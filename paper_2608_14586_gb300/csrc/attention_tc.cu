@@ -3,29 +3,32 @@
 // o[i, h] = sum_{j <= pos0 + i} softmax_j(q_ih . k_gj / sqrt(d_h)) v_gj,  g = h / (H / H_kv)
 //
 // Persistent: one CTA per SM (320 threads, all 512 TMEM columns) walks a list of work units,
-// each a PAIR of query tiles of one head (tile A = 128 query rows, tile B = the next 128),
-// numbered longest first and dealt to the CTAs in a snake so every CTA gets a similar number
-// of key blocks. Both tiles read the same key/value blocks, which are loaded once for the pair.
-//   warp 0      TMA: the pair's two Q tiles, then K and V blocks of 128 keys through a 2-stage K
-//               ring and a 3-stage V ring shared by the two tiles. K/V come from the layer's cache through a 3-D
-//               tensor map whose key extent ends at the context length, so keys past it arrive
-//               as zeros.
-//   warp 1      TMEM allocation; one thread issues, per tile t, S_t = Q_t K^T (M=128, N=128
-//               keys, K=d_h) into TMEM columns [128t, 128t+128) and O_t += P_t V (M=128, N=d_h,
-//               K=128 keys) into TMEM columns [256 + t*d_h, ...), with P_t read from tensor
-//               memory (the softmax writes it as packed bf16 over the first 64 columns of S_t)
-//               and V from shared memory as an MN-major operand. The next S_t is issued right
-//               behind PV_t: one thread's MMAs execute in issue order, so PV_t has read P_t
-//               before S_t is overwritten, and the thread never waits on an MMA.
-//   warps 2..5  softmax of tile A, warps 6..9 of tile B; one thread per query row (TMEM lane):
-//               reads its S row once (tcgen05.ld), masks, takes the row max, writes
-//               P = exp2(s - m) as bf16 into tensor memory (tcgen05.st), keeps the row sum, and
-//               rescales its O row only when the running max grows by more than 2^8 (a stale max
-//               below that is exact arithmetic with values up to 2^8). Each tile is a chain
-//               S -> softmax -> PV -> next S; the two chains of a pair run side by side, so
-//               the tensor core works on one tile while the other's softmax runs. At the end of
-//               a pair each group writes its tile's O / l.
-// Phases of every barrier follow per-CTA block and pair counters. Every wait is bounded.
+// each one query tile (128 rows) of one head, numbered longest first and dealt to the CTAs in
+// a snake so that every CTA gets a similar number of 128-key blocks (with 18 tiles of 32 heads
+// on 152 SMs exactly 36 each). A CTA's key blocks form one sequence g = 0, 1, ... over its
+// units. Tensor memory: three S buffers (columns [0, 128), [128, 256), [256, 384)) and O
+// (d_h columns from 384).
+//   warp 0      TMA: the units' Q tiles into two shared-memory buffers, and K and V blocks of
+//               128 keys through 3- and 2-stage rings, from the layer's cache through 3-D tensor
+//               maps whose key extent ends at the context length (keys past it arrive as zeros,
+//               so stale cache contents never reach P V).
+//   warp 1      TMEM allocation; one thread issues S(g) = Q K_g^T into S buffer g % 3 and
+//               O += P(g) V_g with P(g) (packed bf16 over the first 64 columns of its S buffer)
+//               read from tensor memory and V_g as an MN-major shared-memory operand. S(g + 3)
+//               is issued right behind PV(g): one thread's MMAs execute in issue order, so PV(g)
+//               has read P(g) before S(g + 3) overwrites it. With three S buffers the S of a
+//               block is requested three blocks ahead of its softmax, so the hand-off of P to
+//               this thread and the PV and S that follow stay off the softmax's path.
+//   warps 2..5  softmax, one thread per query row (TMEM lane): reads its S row once
+//               (tcgen05.ld), masks, takes the row max, writes P = exp2(s - m) as bf16 into tensor
+//               memory (tcgen05.st) and keeps the row sum. Only when the running max grows by
+//               more than 2^8 (a stale max below that is exact arithmetic with values up to 2^8)
+//               does it rescale its O row, once PV(g - 1) has completed. At the end of a tile it
+//               hands the row sum to warps 6..9 through shared memory.
+//   warps 6..9  after a tile's last PV: read O, divide by the row sum and store the output rows.
+// Phases of every barrier follow per-CTA block and unit counters; no waiter can fall two
+// phases behind its barrier (each producer of a phase needs the waiter's previous step, or, for
+// the PV barriers waited on only before a rescale, see there). Every wait is bounded.
 #include "common.cuh"
 #include "internal.h"
 
@@ -36,6 +39,9 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kBN = 128;
 constexpr int kThreads = 320;
+constexpr int kSBufs = 3;
+constexpr int kKStages = 3;
+constexpr int kVStages = 2;
 constexpr float kRescaleLog2 = 8.0f;
 
 template <int DH>
@@ -44,24 +50,29 @@ struct AttnCfg {
     static constexpr uint32_t CHUNK = 128 * 64 * 2;  // one [128 rows][64] bf16 chunk
     static constexpr uint32_t Q_BYTES = KCH * CHUNK;
     static constexpr uint32_t KV_BYTES = KCH * CHUNK;
-    static constexpr int K_STAGES = 2;
-    static constexpr int V_STAGES = 3;
-    static constexpr uint32_t OFF_K = 2 * Q_BYTES;  // Q of tile A, then of tile B
-    static constexpr uint32_t OFF_V = OFF_K + K_STAGES * KV_BYTES;
-    static constexpr uint32_t OFF_BAR = OFF_V + V_STAGES * KV_BYTES;
-    static constexpr uint32_t SMEM = OFF_BAR + 256 + 1024;
+    static constexpr uint32_t OFF_K = 2 * Q_BYTES;  // two Q buffers
+    static constexpr uint32_t OFF_V = OFF_K + kKStages * KV_BYTES;
+    static constexpr uint32_t OFF_BAR = OFF_V + kVStages * KV_BYTES;
+    static constexpr uint32_t OFF_L = OFF_BAR + 512;  // row sums handed to the epilogue: [2][128] fp32
+    static constexpr uint32_t SMEM = OFF_L + 2 * kBM * 4 + 1024;
     static constexpr uint32_t TMEM_COLS = 512;
-    static constexpr uint32_t O_COL = 256;  // O of tile t at O_COL + t * DH
+    static constexpr uint32_t O_COL = kSBufs * kBN;
+    static_assert(O_COL + DH <= TMEM_COLS, "tensor memory columns");
+    static_assert(SMEM <= 232448, "shared memory");
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(kBM, kBN);
     static constexpr uint32_t IDESC_O = idesc_bf16_f32_bmn(kBM, DH);
 };
 
 struct Bars {
-    uint64_t q_full, q_free, k_full[2], k_empty[2], v_full[3], v_empty[3];
-    uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];  // per tile
-    uint64_t mma_done;
+    uint64_t k_full[kKStages], k_empty[kKStages], v_full[kVStages], v_empty[kVStages];
+    uint64_t s_full[kSBufs], p_full[kSBufs];  // per S buffer
+    uint64_t q_full[2], q_free[2];            // per Q buffer
+    uint64_t l_full[2], l_free[2];            // per row-sum buffer
+    uint64_t pv_done[2];                      // PV(g) of even / odd g
+    uint64_t o_full, o_free, mma_done;
     uint32_t tmem_slot;
 };
+static_assert(sizeof(Bars) <= 512, "barrier block");
 
 VLA_DEV bool wait_ab(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -73,6 +84,13 @@ VLA_DEV bool wait_ab(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
     return true;
 }
 
+// the same wait in every lane of a warp, true only if every lane's wait succeeded
+VLA_DEV bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+    const bool ok = wait_ab(bar, parity, abort_flag);
+    __syncwarp();
+    return __all_sync(0xFFFFFFFFu, ok);
+}
+
 struct TcAttnArgs {
     int M, H, Hkv, pos0, ctx, ld_out;
     float scale_log2;
@@ -80,29 +98,45 @@ struct TcAttnArgs {
     unsigned* status;
 };
 
-// A pair of query tiles of one head: tile A at rows [m0, m0+128), tile B at [m0+128, m0+256)
-// (absent when m0 + 128 >= M), and the key blocks each needs.
-struct Pair {
-    int h, g, m0, n[2];  // n[1] == 0: no tile B
+// A query tile of one head: rows [m0, m0 + 128) (clipped to M) of head h, KV head g, and the
+// n key blocks of 128 it attends to.
+struct Unit {
+    int h, g, m0, n;
 };
 
-// The CTA's k-th pair, or false. Pairs are numbered longest first (every head of the latest
-// pair of query tiles, then the next, ...) and dealt to the persistent CTAs in a snake
+// The CTA's k-th unit, or false. Units are numbered longest first (every head of the last
+// query tile, then of the one before, ...) and dealt to the persistent CTAs in a snake
 // (round r: CTA c takes unit r*G + c on even rounds, (r+1)*G - 1 - c on odd ones).
-VLA_DEV bool cta_pair(int k, int num_p, const TcAttnArgs& a, Pair& p) {
+VLA_DEV bool cta_unit(int k, int num_t, const TcAttnArgs& a, Unit& u) {
     const int G = gridDim.x, c = blockIdx.x;
     const int idx = (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
-    if (idx >= num_p * a.H) return false;
-    const int pm = num_p - 1 - idx / a.H;
-    p.h = idx % a.H;
-    p.g = p.h / (a.H / a.Hkv);
-    p.m0 = pm * 2 * kBM;
-    for (int t = 0; t < 2; ++t) {
-        const int r0 = p.m0 + t * kBM;
-        p.n[t] = r0 < a.M ? (a.pos0 + min(r0 + kBM, a.M) + kBN - 1) / kBN : 0;
-    }
+    if (idx >= num_t * a.H) return false;
+    const int tm = num_t - 1 - idx / a.H;
+    u.h = idx % a.H;
+    u.g = u.h / (a.H / a.Hkv);
+    u.m0 = tm * kBM;
+    u.n = (a.pos0 + min(u.m0 + kBM, a.M) + kBN - 1) / kBN;
     return true;
 }
+
+// A position (unit k, block j of it) in the CTA's block sequence.
+struct Cursor {
+    int k, j;
+    Unit u;
+    bool valid;
+    VLA_DEV void start(int num_t, const TcAttnArgs& a) {
+        k = 0;
+        j = 0;
+        valid = cta_unit(0, num_t, a, u);
+    }
+    VLA_DEV void next(int num_t, const TcAttnArgs& a) {
+        if (++j == u.n) {
+            j = 0;
+            ++k;
+            valid = cta_unit(k, num_t, a, u);
+        }
+    }
+};
 
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -114,25 +148,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
     uint8_t* smem = smem_raw + pad;
     Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
+    float* lbuf = reinterpret_cast<float*>(smem + C::OFF_L);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_p = (a.M + 2 * kBM - 1) / (2 * kBM);
+    const int num_t = (a.M + kBM - 1) / kBM;
 
     if (threadIdx.x == 0) {
-        mbar_init(&bars->q_full, 1);
-        mbar_init(&bars->q_free, 1);
-        for (int b = 0; b < 3; ++b) {
+        for (int b = 0; b < kKStages; ++b) {
+            mbar_init(&bars->k_full[b], 1);
+            mbar_init(&bars->k_empty[b], 1);
+        }
+        for (int b = 0; b < kVStages; ++b) {
             mbar_init(&bars->v_full[b], 1);
             mbar_init(&bars->v_empty[b], 1);
         }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(&bars->k_full[b], 1);
-            mbar_init(&bars->k_empty[b], 1);
+        for (int b = 0; b < kSBufs; ++b) {
             mbar_init(&bars->s_full[b], 1);
             mbar_init(&bars->p_full[b], 128);
-            mbar_init(&bars->pv_done[b], 1);
-            mbar_init(&bars->o_free[b], 128);
         }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&bars->q_full[b], 1);
+            mbar_init(&bars->q_free[b], 1);
+            mbar_init(&bars->l_full[b], 128);
+            mbar_init(&bars->l_free[b], 128);
+            mbar_init(&bars->pv_done[b], 1);
+        }
+        mbar_init(&bars->o_full, 1);
+        mbar_init(&bars->o_free, 128);
         mbar_init(&bars->mma_done, 1);
         s_abort = 0;
         fence_barrier_init();
@@ -156,68 +198,67 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer ----------------
-            // ring slot of global block n: n % 2, phase (n / 2) & 1 (K and V alike)
+            // Q of unit k into Q buffer k % 2, K(g) into K slot g % 3 and V(g) into V slot g % 2,
+            // each in order; whichever has a free slot goes next
             bool ok = true;
-            uint32_t issued_k = 0, issued_v = 0, ph_k = 0, ph_v = 0;
-            bool issued_q = false;
-            uint32_t ph_q = 0;
-            uint32_t nk = 0, nv = 0;  // K / V blocks issued so far (all pairs)
-            Pair p;
+            Cursor ck, cv;
+            ck.start(num_t, a);
+            cv.start(num_t, a);
+            int kq = 0;
+            Unit uq;
+            bool q_left = cta_unit(0, num_t, a, uq);
+            uint32_t nk = 0, nv = 0;
+            uint32_t issued_k = 0, ph_k = 0, issued_v = 0, ph_v = 0, issued_q = 0, ph_q = 0;
             long long t0 = clock64();
-            for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
-                if (!wait_ab(&bars->q_free, ((uint32_t)k & 1u) ^ 1u, &s_abort)) {
+            while (ck.valid || cv.valid || q_left) {
+                bool progressed = false;
+                if (q_left) {
+                    const uint32_t b = (uint32_t)kq & 1u, n = (uint32_t)kq >> 1;
+                    if (mbar_try_wait(&bars->q_free[b], (n & 1u) ^ 1u)) {
+                        mbar_arrive_expect_tx(&bars->q_full[b], C::Q_BYTES);
+                        for (int c = 0; c < C::KCH; ++c)
+                            tma_load_2d(smem + b * C::Q_BYTES + c * C::CHUNK, &tmQ, &bars->q_full[b],
+                                        uq.h * DH + c * 64, uq.m0);
+                        issued_q |= 1u << b;
+                        ph_q = (ph_q & ~(1u << b)) | ((n & 1u) << b);
+                        ++kq;
+                        q_left = cta_unit(kq, num_t, a, uq);
+                        progressed = true;
+                    }
+                }
+                if (ck.valid) {
+                    const uint32_t b = nk % kKStages, n = nk / kKStages;
+                    if (mbar_try_wait(&bars->k_empty[b], (n & 1u) ^ 1u)) {
+                        mbar_arrive_expect_tx(&bars->k_full[b], C::KV_BYTES);
+                        for (int c = 0; c < C::KCH; ++c)
+                            tma_load_3d(smem + C::OFF_K + b * C::KV_BYTES + c * C::CHUNK, &tmK, &bars->k_full[b],
+                                        c * 64, ck.j * kBN, ck.u.g);
+                        issued_k |= 1u << b;
+                        ph_k = (ph_k & ~(1u << b)) | ((n & 1u) << b);
+                        ++nk;
+                        ck.next(num_t, a);
+                        progressed = true;
+                    }
+                }
+                if (cv.valid) {
+                    const uint32_t b = nv % kVStages, n = nv / kVStages;
+                    if (mbar_try_wait(&bars->v_empty[b], (n & 1u) ^ 1u)) {
+                        mbar_arrive_expect_tx(&bars->v_full[b], C::KV_BYTES);
+                        for (int c = 0; c < C::KCH; ++c)
+                            tma_load_3d(smem + C::OFF_V + b * C::KV_BYTES + c * C::CHUNK, &tmV, &bars->v_full[b],
+                                        c * 64, cv.j * kBN, cv.u.g);
+                        issued_v |= 1u << b;
+                        ph_v = (ph_v & ~(1u << b)) | ((n & 1u) << b);
+                        ++nv;
+                        cv.next(num_t, a);
+                        progressed = true;
+                    }
+                }
+                if (progressed) {
+                    t0 = clock64();
+                } else if (s_abort || clock64() - t0 > kWaitBudgetCycles) {
                     ok = false;
                     break;
-                }
-                const int ntiles = p.n[1] > 0 ? 2 : 1;
-                mbar_arrive_expect_tx(&bars->q_full, C::Q_BYTES * ntiles);
-                for (int t = 0; t < ntiles; ++t)
-                    for (int c = 0; c < C::KCH; ++c)
-                        tma_load_2d(smem + t * C::Q_BYTES + c * C::CHUNK, &tmQ, &bars->q_full, p.h * DH + c * 64,
-                                    p.m0 + t * kBM);
-                issued_q = true;
-                ph_q = (uint32_t)k & 1u;
-                const int nmax = max(p.n[0], p.n[1]);
-                int jk = 0, jv = 0;
-                t0 = clock64();
-                while (jk < nmax || jv < nmax) {
-                    bool progressed = false;
-                    if (jk < nmax) {
-                        const int b = nk & 1;
-                        const uint32_t n = nk >> 1;
-                        if (mbar_try_wait(&bars->k_empty[b], (n & 1u) ^ 1u)) {
-                            mbar_arrive_expect_tx(&bars->k_full[b], C::KV_BYTES);
-                            for (int c = 0; c < C::KCH; ++c)
-                                tma_load_3d(smem + C::OFF_K + b * C::KV_BYTES + c * C::CHUNK, &tmK, &bars->k_full[b],
-                                            c * 64, jk * kBN, p.g);
-                            issued_k |= 1u << b;
-                            ph_k = (ph_k & ~(1u << b)) | ((n & 1u) << b);
-                            ++jk;
-                            ++nk;
-                            progressed = true;
-                        }
-                    }
-                    if (jv < nmax) {  // V runs ahead of K as far as its ring allows
-                        const int b = (int)(nv % 3u);
-                        const uint32_t n = nv / 3u;
-                        if (mbar_try_wait(&bars->v_empty[b], (n & 1u) ^ 1u)) {
-                            mbar_arrive_expect_tx(&bars->v_full[b], C::KV_BYTES);
-                            for (int c = 0; c < C::KCH; ++c)
-                                tma_load_3d(smem + C::OFF_V + b * C::KV_BYTES + c * C::CHUNK, &tmV, &bars->v_full[b],
-                                            c * 64, jv * kBN, p.g);
-                            issued_v |= 1u << b;
-                            ph_v = (ph_v & ~(1u << b)) | ((n & 1u) << b);
-                            ++jv;
-                            ++nv;
-                            progressed = true;
-                        }
-                    }
-                    if (progressed) {
-                        t0 = clock64();
-                    } else if (s_abort || clock64() - t0 > kWaitBudgetCycles) {
-                        ok = false;
-                        break;
-                    }
                 }
             }
             if (!ok) {
@@ -225,89 +266,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                 set_status(a.status, kDevTimeout);
             }
             // every copy this thread issued lands before the CTA can exit
-            if (issued_q) mbar_wait(&bars->q_full, ph_q);
-            for (int b = 0; b < 3; ++b) {
-                if (b < 2 && (issued_k & (1u << b))) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
+            for (int b = 0; b < 2; ++b)
+                if (issued_q & (1u << b)) mbar_wait(&bars->q_full[b], (ph_q >> b) & 1u);
+            for (int b = 0; b < kKStages; ++b)
+                if (issued_k & (1u << b)) mbar_wait(&bars->k_full[b], (ph_k >> b) & 1u);
+            for (int b = 0; b < kVStages; ++b)
                 if (issued_v & (1u << b)) mbar_wait(&bars->v_full[b], (ph_v >> b) & 1u);
-            }
         }
     } else if (warp == 1) {
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
             bool ok = true;
-            uint32_t gt[2] = {0, 0};  // blocks of tile slot t so far (S, P, PV phases)
-            uint32_t et[2] = {0, 0};  // pairs in which tile slot t existed (O phases)
-            uint32_t nkv = 0;         // K/V blocks so far (ring phases)
-            auto issue_s = [&](int t, uint32_t n, uint32_t sQ) {
-                const uint32_t sK = smem_u32(smem + C::OFF_K + (n & 1) * C::KV_BYTES);
+            Cursor cs;  // the next S to issue
+            cs.start(num_t, a);
+            uint32_t gs = 0;  // S issued so far
+            // S(gs) = Q K^T into S buffer gs % 3, once the unit's Q and K_gs are loaded
+            auto issue_s = [&]() -> bool {
+                if (!cs.valid) return true;
+                const uint32_t qb = (uint32_t)cs.k & 1u;
+                const uint32_t kb = gs % kKStages;
+                if ((cs.j == 0 && !wait_ab(&bars->q_full[qb], ((uint32_t)cs.k >> 1) & 1u, &s_abort)) ||
+                    !wait_ab(&bars->k_full[kb], (gs / kKStages) & 1u, &s_abort))
+                    return false;
+                tc_fence_after();
+                const uint32_t sQ = smem_u32(smem + qb * C::Q_BYTES);
+                const uint32_t sK = smem_u32(smem + C::OFF_K + kb * C::KV_BYTES);
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk) {
                     const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
                     const uint64_t bd = sw128_kmajor_desc(sK + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                    umma_bf16_ss(tmem + t * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
+                    umma_bf16_ss(tmem + (gs % kSBufs) * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(&bars->s_full[t]);
+                umma_commit(&bars->s_full[gs % kSBufs]);
+                umma_commit(&bars->k_empty[kb]);
+                if (cs.j == cs.u.n - 1) umma_commit(&bars->q_free[qb]);  // the unit's last S
+                ++gs;
+                cs.next(num_t, a);
+                return true;
             };
-            Pair p;
-            for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
-                const int nmax = max(p.n[0], p.n[1]);
-                if (!wait_ab(&bars->q_full, (uint32_t)k & 1u, &s_abort) ||
-                    !wait_ab(&bars->k_full[nkv & 1], (nkv >> 1) & 1u, &s_abort)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                // S of block 0 for both tiles: their columns hold the previous pair's last P,
-                // read by a PV issued before (issue order, as below)
-                for (int t = 0; t < 2; ++t)
-                    if (p.n[t] > 0) issue_s(t, nkv, smem_u32(smem + t * C::Q_BYTES));
-                umma_commit(&bars->k_empty[nkv & 1]);
-                if (nmax == 1) umma_commit(&bars->q_free);
-                for (int j = 0; j < nmax && ok; ++j) {
-                    const uint32_t n = nkv + j;
-                    const uint32_t vs = n % 3u;  // V ring slot of block n, phase (n / 3) & 1
-                    if (!wait_ab(&bars->v_full[vs], (n / 3u) & 1u, &s_abort) ||
-                        (j + 1 < nmax && !wait_ab(&bars->k_full[(n + 1) & 1], ((n + 1) >> 1) & 1u, &s_abort))) {
+            for (int i = 0; i < kSBufs && ok; ++i) ok = issue_s();
+            uint32_t g = 0;  // PV issued so far
+            Unit u;
+            for (int k = 0; ok && cta_unit(k, num_t, a, u); ++k) {
+                for (int j = 0; j < u.n; ++j, ++g) {
+                    const uint32_t sb = g % kSBufs, vb = g % kVStages;
+                    if (!wait_ab(&bars->p_full[sb], (g / kSBufs) & 1u, &s_abort) ||
+                        (j == 0 && !wait_ab(&bars->o_free, ((uint32_t)k & 1u) ^ 1u, &s_abort)) ||
+                        !wait_ab(&bars->v_full[vb], (g / kVStages) & 1u, &s_abort)) {
                         ok = false;
                         break;
                     }
-                    for (int t = 0; t < 2 && ok; ++t) {
-                        if (j >= p.n[t]) continue;
-                        if (!wait_ab(&bars->p_full[t], gt[t] & 1u, &s_abort) ||
-                            (j == 0 && !wait_ab(&bars->o_free[t], (et[t] & 1u) ^ 1u, &s_abort))) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint32_t sV = smem_u32(smem + C::OFF_V + vs * C::KV_BYTES);
+                    tc_fence_after();
+                    const uint32_t sV = smem_u32(smem + C::OFF_V + vb * C::KV_BYTES);
 #pragma unroll
-                        for (int kk = 0; kk < kBN / 16; ++kk) {
-                            const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
-                            umma_bf16_ts(tmem + C::O_COL + t * DH, tmem + t * kBN + kk * 8, bd, C::IDESC_O,
-                                         (j > 0 || kk > 0) ? 1u : 0u);
-                        }
-                        // the block's last PV: V_j's slot is free once it completes (committed
-                        // before the next S, so the producer can refill it while that S runs)
-                        if (t == 1 || j >= p.n[1]) umma_commit(&bars->v_empty[vs]);
-                        // The next S of this tile overwrites P_t in the same columns. It is issued
-                        // right behind the PV that reads P_t: the tensor core executes one thread's
-                        // MMAs in issue order, so the PV's operand reads precede the S's writes.
-                        // Its commit also tells the softmax that PV_t has completed (O_t may be
-                        // rescaled).
-                        if (j + 1 < p.n[t]) issue_s(t, n + 1, smem_u32(smem + t * C::Q_BYTES));
-                        else umma_commit(&bars->pv_done[t]);  // the tile's last PV: O_t is final
-                        ++gt[t];
+                    for (int kk = 0; kk < kBN / 16; ++kk) {
+                        const uint64_t bd = sw128_mnmajor_desc(sV + kk * 16 * 128, C::CHUNK);
+                        umma_bf16_ts(tmem + C::O_COL, tmem + sb * kBN + kk * 8, bd, C::IDESC_O,
+                                     (j > 0 || kk > 0) ? 1u : 0u);
                     }
-                    if (!ok) break;
-                    if (j + 1 < nmax) {
-                        umma_commit(&bars->k_empty[(n + 1) & 1]);
-                        if (j + 2 == nmax) umma_commit(&bars->q_free);  // the pair's last S was just issued
+                    umma_commit(&bars->v_empty[vb]);
+                    umma_commit(&bars->pv_done[g & 1u]);
+                    if (j == u.n - 1) umma_commit(&bars->o_full);  // O of the unit is final
+                    // S(g + 3) reuses the buffer of P(g): issued after the PV that reads it
+                    if (!issue_s()) {
+                        ok = false;
+                        break;
                     }
                 }
-                if (!ok) break;
-                for (int t = 0; t < 2; ++t)
-                    if (p.n[t] > 0) ++et[t];
-                nkv += nmax;
             }
             if (!ok) {
                 s_abort = 1;
@@ -317,34 +342,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(&bars->mma_done);
             mbar_wait(&bars->mma_done, 0);
         }
-    } else {
-        // ---------------- softmax / correction / epilogue: tile A (warps 2..5), B (6..9) ----------------
-        const int t = (warp - 2) >> 2;
+    } else if (warp < 6) {
+        // ---------------- softmax (warps 2..5) ----------------
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-        const uint32_t scol = (uint32_t)t * kBN;
-        const uint32_t ocol = C::O_COL + (uint32_t)t * DH;
         bool ok = true;
-        uint32_t g = 0;   // blocks of this tile slot so far (S and P phases)
-        uint32_t np = 0;  // pairs in which this tile slot existed (final-PV phases)
-        Pair p;
-        for (int k = 0; ok && cta_pair(k, num_p, a, p); ++k) {
-            if (p.n[t] == 0) continue;  // no tile B in this pair
-            const int m0 = p.m0 + t * kBM;
-            const int qpos = a.pos0 + m0 + row;
-            const int min_qpos = a.pos0 + m0;
+        uint32_t g = 0;  // blocks so far (S buffer phases)
+        Unit u;
+        for (int k = 0; ok && cta_unit(k, num_t, a, u); ++k) {
+            const int qpos = a.pos0 + u.m0 + row;
+            const int min_qpos = a.pos0 + u.m0;
             float m_run = -INFINITY, l_run = 0.f;
-            for (int j = 0; j < p.n[t]; ++j) {
+            for (int j = 0; j < u.n; ++j, ++g) {
+                const uint32_t scol = (g % kSBufs) * kBN;
                 uint32_t sr[kBN];
                 float m_new = m_run;
                 bool need = false;
                 {
                     const int kb = j * kBN;
                     const bool need_mask = (kb + kBN - 1 > min_qpos) || (kb + kBN > a.ctx);
-                    ok = wait_ab(&bars->s_full[t], g & 1u, &s_abort);
-                    __syncwarp();
-                    if (!__all_sync(0xFFFFFFFFu, ok)) {
+                    if (!warp_wait(&bars->s_full[g % kSBufs], (g / kSBufs) & 1u, &s_abort)) {
                         ok = false;
                         break;
                     }
@@ -381,7 +399,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float corr = need ? ex2_approx(m_run - m_new) : 1.f;
                     l_run *= corr;
                     const bool warp_need = __any_sync(0xFFFFFFFFu, need);
-                    // P = exp2(s * scale - m) as packed bf16 over the first 64 columns of S
+                    // P = exp2(s * scale - m) as packed bf16 over the first 64 columns of S,
                     // two columns per instruction for the scaling and the row sum (packed fp32)
                     const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
                     const float2 nm2 = make_float2(-m_new, -m_new);
@@ -405,51 +423,82 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_wait_st();
                     l_run += (ls[0].x + ls[1].x) + (ls[0].y + ls[1].y);
                     if (warp_need) {
-                        // PV of the previous block has completed: this block's S was issued after it
+                        // O is rescaled once PV(g - 1) has completed (it commits to the barrier
+                        // of its parity). PV(g - 3) has completed (S(g), seen above, was issued
+                        // after it) and PV(g + 1) cannot start before P(g + 1) exists, so among
+                        // the PVs of that parity only PV(g - 1) may be outstanding: the barrier
+                        // is exactly one phase short or complete, though this wait is skipped
+                        // whenever no rescale is needed.
+                        if (!warp_wait(&bars->pv_done[(g - 1) & 1u], ((g - 1) >> 1) & 1u, &s_abort)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
 #pragma unroll 1
                         for (int c = 0; c < DH / 32; ++c) {
                             uint32_t r[32];
-                            tmem_ld32(trow + ocol + c * 32, r);
+                            tmem_ld32(trow + C::O_COL + c * 32, r);
 #pragma unroll
                             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * corr);
-                            tmem_st32(trow + ocol + c * 32, r);
+                            tmem_st32(trow + C::O_COL + c * 32, r);
                         }
                     }
                     tc_fence_before();
-                    mbar_arrive(&bars->p_full[t]);
+                    mbar_arrive(&bars->p_full[g % kSBufs]);
                     m_run = m_new;
-                    ++g;
                 }
             }
             if (!ok) break;
-            // epilogue of this tile: after its last PV
-            ok = wait_ab(&bars->pv_done[t], np & 1u, &s_abort);
-            ++np;
-            __syncwarp();
-            if (!__all_sync(0xFFFFFFFFu, ok)) {
+            // the row sum to the epilogue thread of the same row
+            const uint32_t lb = (uint32_t)k & 1u;
+            if (!warp_wait(&bars->l_free[lb], (((uint32_t)k >> 1) & 1u) ^ 1u, &s_abort)) {
+                ok = false;
+                break;
+            }
+            lbuf[lb * kBM + row] = l_run;
+            mbar_arrive(&bars->l_full[lb]);
+        }
+        if (!ok) {
+            s_abort = 1;
+            set_status(a.status, kDevTimeout);
+        }
+    } else {
+        // ---------------- output epilogue (warps 6..9) ----------------
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;
+        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+        bool ok = true;
+        Unit u;
+        for (int k = 0; ok && cta_unit(k, num_t, a, u); ++k) {
+            const uint32_t lb = (uint32_t)k & 1u;
+            if (!warp_wait(&bars->o_full, (uint32_t)k & 1u, &s_abort) ||
+                !warp_wait(&bars->l_full[lb], ((uint32_t)k >> 1) & 1u, &s_abort)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-            const bool row_ok = (m0 + row) < a.M;
-            bf16* orow = a.out + (size_t)(m0 + row) * a.ld_out + p.h * DH;
-#pragma unroll 1
-            for (int c = 0; c < DH / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(trow + ocol + c * 32, r);
-                if (!row_ok) continue;
-                uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+            const float l = lbuf[lb * kBM + row];
+            uint32_t o[DH];
+            if constexpr (DH == 128) {
+                tmem_ld128(trow + C::O_COL, o);
+            } else {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    dst[q] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * q]) * inv, __uint_as_float(r[8 * q + 1]) * inv),
-                                        pack_bf16x2(__uint_as_float(r[8 * q + 2]) * inv, __uint_as_float(r[8 * q + 3]) * inv),
-                                        pack_bf16x2(__uint_as_float(r[8 * q + 4]) * inv, __uint_as_float(r[8 * q + 5]) * inv),
-                                        pack_bf16x2(__uint_as_float(r[8 * q + 6]) * inv, __uint_as_float(r[8 * q + 7]) * inv));
-                }
+                for (int c = 0; c < DH / 32; ++c)
+                    tmem_ld32(trow + C::O_COL + c * 32, *reinterpret_cast<uint32_t(*)[32]>(o + 32 * c));
             }
             tc_fence_before();
-            mbar_arrive(&bars->o_free[t]);
+            mbar_arrive(&bars->o_free);
+            mbar_arrive(&bars->l_free[lb]);
+            const float inv = l > 0.f ? 1.f / l : 0.f;
+            if (u.m0 + row < a.M) {
+                uint4* dst = reinterpret_cast<uint4*>(a.out + (size_t)(u.m0 + row) * a.ld_out + u.h * DH);
+#pragma unroll
+                for (int q = 0; q < DH / 8; ++q)
+                    dst[q] = make_uint4(pack_bf16x2(__uint_as_float(o[8 * q]) * inv, __uint_as_float(o[8 * q + 1]) * inv),
+                                        pack_bf16x2(__uint_as_float(o[8 * q + 2]) * inv, __uint_as_float(o[8 * q + 3]) * inv),
+                                        pack_bf16x2(__uint_as_float(o[8 * q + 4]) * inv, __uint_as_float(o[8 * q + 5]) * inv),
+                                        pack_bf16x2(__uint_as_float(o[8 * q + 6]) * inv, __uint_as_float(o[8 * q + 7]) * inv));
+            }
         }
         if (!ok) {
             s_abort = 1;
@@ -488,14 +537,14 @@ cudaError_t launch_dh(const AttnPrefillParams& p, unsigned* status, cudaStream_t
     a.scale_log2 = p.scale_log2;
     a.out = p.out;
     a.status = status;
-    // persistent: one CTA per SM (tensor-memory kernels get one per SM), each walking its pairs
+    // persistent: one CTA per SM (tensor-memory kernels get one per SM), each walking its units
     static const int sms = [] {
         int dev = 0, n = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
         return n > 0 ? n : 1;
     }();
-    const int units = ((p.M + 2 * kBM - 1) / (2 * kBM)) * p.H;
+    const int units = ((p.M + kBM - 1) / kBM) * p.H;
     const dim3 grid(units < sms ? units : sms);
     return launch_ex(attn_prefill_tc_kernel<DH>, grid, dim3(kThreads), C::SMEM, stream, pdl, tq, tk, tv, a);
 }
