@@ -55,7 +55,7 @@ def test_barrier_and_max_over_ranks():
 
 def test_reference_arm_prints_on_rank_zero_only():
     """Rank 1 of the reference arm exits 0 without work or output; rank 0 prints the line.
-    Rank 0's oracle run is stubbed here (its own timing is covered on the GPU machine)."""
+    Rank 0's oracle run is stubbed here (the full reference arm runs it in the bench)."""
     code = textwrap.dedent("""
         import json, sys
         import bench
