@@ -44,6 +44,8 @@ def test_gemm_matches_definition(vla_lib, M, N, K):
     (96, 8, 4, 64, 3),        # GQA group 2
     (150, 16, 2, 128, 9),     # GQA group 8, ragged M, continuing context
     (1024, 32, 8, 128, 0),    # 7B shape
+    (64, 320, 8, 64, 0),      # more one-block query tiles than SMs: consecutive tiny units per CTA
+    (100, 160, 16, 128, 300), # long continuing context, four key blocks per ragged query tile
 ])
 def test_attention_prefill_matches_oracle(vla_lib, M, H, Hkv, dh, pos0):
     import torch
