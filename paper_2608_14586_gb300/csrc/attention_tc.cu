@@ -2,7 +2,7 @@
 //
 // o[i, h] = sum_{j <= pos0 + i} softmax_j(q_ih . k_gj / sqrt(d_h)) v_gj,  g = h / (H / H_kv)
 //
-// Persistent: one CTA per SM (320 threads, all 512 TMEM columns) walks a list of work units,
+// Persistent: one CTA per SM (352 threads, all 512 TMEM columns) walks a list of work units,
 // each one query tile (128 rows) of one head, numbered longest first and dealt to the CTAs in
 // a snake so that every CTA gets a similar number of 128-key blocks (with 18 tiles of 32 heads
 // on 152 SMs exactly 36 each). A CTA's key blocks form one sequence g = 0, 1, ... over its
@@ -12,13 +12,14 @@
 //               128 keys through 3- and 2-stage rings, from the layer's cache through 3-D tensor
 //               maps whose key extent ends at the context length (keys past it arrive as zeros,
 //               so stale cache contents never reach P V).
-//   warp 1      TMEM allocation; one thread issues S(g) = Q K_g^T into S buffer g % 3 and
-//               O += P(g) V_g with P(g) (packed bf16 over the first 64 columns of its S buffer)
-//               read from tensor memory and V_g as an MN-major shared-memory operand. S(g + 3)
-//               is issued right behind PV(g): one thread's MMAs execute in issue order, so PV(g)
-//               has read P(g) before S(g + 3) overwrites it. With three S buffers the S of a
-//               block is requested three blocks ahead of its softmax, so the hand-off of P to
-//               this thread and the PV and S that follow stay off the softmax's path.
+//   warp 1      TMEM allocation; one thread issues O += P(g) V_g with P(g) (packed bf16 over the
+//               first 64 columns of S buffer g % 3) read from tensor memory and V_g as an
+//               MN-major shared-memory operand, and commits the PV's completion on the barrier
+//               of that buffer.
+//   warp 10     one thread issues S(g) = Q K_g^T into S buffer g % 3 once PV(g - 3), the last
+//               reader of that buffer, has completed. The S of a block is requested three blocks
+//               ahead of its softmax, and with two issuing threads one's waits overlap the
+//               other's issue, so the tensor core is fed from both.
 //   warps 2..5  softmax, one thread per query row (TMEM lane): reads its S row once
 //               (tcgen05.ld), masks, takes the row max, writes P = exp2(s - m) as bf16 into tensor
 //               memory (tcgen05.st) and keeps the row sum. Only when the running max grows by
@@ -28,7 +29,7 @@
 //   warps 6..9  after a tile's last PV: read O, divide by the row sum and store the output rows.
 // Phases of every barrier follow per-CTA block and unit counters; no waiter can fall two
 // phases behind its barrier (each producer of a phase needs the waiter's previous step, or, for
-// the PV barriers waited on only before a rescale, see there). Every wait is bounded.
+// the PV barriers the softmax waits on only before a rescale, see there). Every wait is bounded.
 #include "common.cuh"
 #include "internal.h"
 
@@ -38,7 +39,7 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;  // + warp 10: the S issuer
 constexpr int kSBufs = 3;
 constexpr int kKStages = 3;
 constexpr int kVStages = 2;
@@ -68,8 +69,8 @@ struct Bars {
     uint64_t s_full[kSBufs], p_full[kSBufs];  // per S buffer
     uint64_t q_full[2], q_free[2];            // per Q buffer
     uint64_t l_full[2], l_free[2];            // per row-sum buffer
-    uint64_t pv_done[2];                      // PV(g) of even / odd g
-    uint64_t o_full, o_free, mma_done;
+    uint64_t pv_done[kSBufs];                 // PV(g) by g % 3 (the S buffer it read)
+    uint64_t o_full, o_free, mma_done, s_done;
     uint32_t tmem_slot;
 };
 static_assert(sizeof(Bars) <= 512, "barrier block");
@@ -171,11 +172,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&bars->q_free[b], 1);
             mbar_init(&bars->l_full[b], 128);
             mbar_init(&bars->l_free[b], 128);
-            mbar_init(&bars->pv_done[b], 1);
         }
+        for (int b = 0; b < kSBufs; ++b) mbar_init(&bars->pv_done[b], 1);
         mbar_init(&bars->o_full, 1);
         mbar_init(&bars->o_free, 128);
         mbar_init(&bars->mma_done, 1);
+        mbar_init(&bars->s_done, 1);
         s_abort = 0;
         fence_barrier_init();
     }
@@ -275,36 +277,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            // ---------------- MMA issuer ----------------
+            // ---------------- PV issuer ----------------
             bool ok = true;
-            Cursor cs;  // the next S to issue
-            cs.start(num_t, a);
-            uint32_t gs = 0;  // S issued so far
-            // S(gs) = Q K^T into S buffer gs % 3, once the unit's Q and K_gs are loaded
-            auto issue_s = [&]() -> bool {
-                if (!cs.valid) return true;
-                const uint32_t qb = (uint32_t)cs.k & 1u;
-                const uint32_t kb = gs % kKStages;
-                if ((cs.j == 0 && !wait_ab(&bars->q_full[qb], ((uint32_t)cs.k >> 1) & 1u, &s_abort)) ||
-                    !wait_ab(&bars->k_full[kb], (gs / kKStages) & 1u, &s_abort))
-                    return false;
-                tc_fence_after();
-                const uint32_t sQ = smem_u32(smem + qb * C::Q_BYTES);
-                const uint32_t sK = smem_u32(smem + C::OFF_K + kb * C::KV_BYTES);
-#pragma unroll
-                for (int kk = 0; kk < DH / 16; ++kk) {
-                    const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                    const uint64_t bd = sw128_kmajor_desc(sK + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
-                    umma_bf16_ss(tmem + (gs % kSBufs) * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
-                }
-                umma_commit(&bars->s_full[gs % kSBufs]);
-                umma_commit(&bars->k_empty[kb]);
-                if (cs.j == cs.u.n - 1) umma_commit(&bars->q_free[qb]);  // the unit's last S
-                ++gs;
-                cs.next(num_t, a);
-                return true;
-            };
-            for (int i = 0; i < kSBufs && ok; ++i) ok = issue_s();
             uint32_t g = 0;  // PV issued so far
             Unit u;
             for (int k = 0; ok && cta_unit(k, num_t, a, u); ++k) {
@@ -325,13 +299,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      (j > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(&bars->v_empty[vb]);
-                    umma_commit(&bars->pv_done[g & 1u]);
+                    umma_commit(&bars->pv_done[sb]);  // the S issuer reuses buffer sb after it
                     if (j == u.n - 1) umma_commit(&bars->o_full);  // O of the unit is final
-                    // S(g + 3) reuses the buffer of P(g): issued after the PV that reads it
-                    if (!issue_s()) {
-                        ok = false;
-                        break;
-                    }
                 }
             }
             if (!ok) {
@@ -341,6 +310,46 @@ __global__ void __launch_bounds__(kThreads, 1)
             // all MMAs issued by this thread retire before TMEM can be released
             umma_commit(&bars->mma_done);
             mbar_wait(&bars->mma_done, 0);
+        }
+    } else if (warp == 10) {
+        if (lane == 0) {
+            // ---------------- S issuer ----------------
+            // S(g) into buffer g % 3 once PV(g - 3), the last reader of that buffer, has
+            // completed (its commit on pv_done[g % 3]; every phase waited in order, and the next
+            // phase needs S(g) itself, so the wait is exact), and the unit's Q and K_g are in
+            bool ok = true;
+            Cursor cs;
+            cs.start(num_t, a);
+            for (uint32_t gs = 0; ok && cs.valid; ++gs) {
+                const uint32_t qb = (uint32_t)cs.k & 1u;
+                const uint32_t kb = gs % kKStages;
+                if ((gs >= (uint32_t)kSBufs &&
+                     !wait_ab(&bars->pv_done[gs % kSBufs], ((gs / kSBufs) - 1u) & 1u, &s_abort)) ||
+                    (cs.j == 0 && !wait_ab(&bars->q_full[qb], ((uint32_t)cs.k >> 1) & 1u, &s_abort)) ||
+                    !wait_ab(&bars->k_full[kb], (gs / kKStages) & 1u, &s_abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sQ = smem_u32(smem + qb * C::Q_BYTES);
+                const uint32_t sK = smem_u32(smem + C::OFF_K + kb * C::KV_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < DH / 16; ++kk) {
+                    const uint64_t ad = sw128_kmajor_desc(sQ + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
+                    const uint64_t bd = sw128_kmajor_desc(sK + (kk >> 2) * C::CHUNK) + 2 * (kk & 3);
+                    umma_bf16_ss(tmem + (gs % kSBufs) * kBN, ad, bd, C::IDESC_S, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&bars->s_full[gs % kSBufs]);
+                umma_commit(&bars->k_empty[kb]);
+                if (cs.j == cs.u.n - 1) umma_commit(&bars->q_free[qb]);  // the unit's last S
+                cs.next(num_t, a);
+            }
+            if (!ok) {
+                s_abort = 1;
+                set_status(a.status, kDevTimeout);
+            }
+            umma_commit(&bars->s_done);
+            mbar_wait(&bars->s_done, 0);
         }
     } else if (warp < 6) {
         // ---------------- softmax (warps 2..5) ----------------
@@ -424,12 +433,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     l_run += (ls[0].x + ls[1].x) + (ls[0].y + ls[1].y);
                     if (warp_need) {
                         // O is rescaled once PV(g - 1) has completed (it commits to the barrier
-                        // of its parity). PV(g - 3) has completed (S(g), seen above, was issued
-                        // after it) and PV(g + 1) cannot start before P(g + 1) exists, so among
-                        // the PVs of that parity only PV(g - 1) may be outstanding: the barrier
-                        // is exactly one phase short or complete, though this wait is skipped
-                        // whenever no rescale is needed.
-                        if (!warp_wait(&bars->pv_done[(g - 1) & 1u], ((g - 1) >> 1) & 1u, &s_abort)) {
+                        // of its S buffer). PV(g - 3) has completed (S(g), seen above, was issued
+                        // after it, so PV(g - 4) too) and PV(g + 2) cannot start before P(g + 2)
+                        // exists, so among the PVs of that buffer only PV(g - 1) may be
+                        // outstanding: the barrier is exactly one phase short or complete,
+                        // though this wait is skipped whenever no rescale is needed.
+                        if (!warp_wait(&bars->pv_done[(g - 1) % kSBufs], ((g - 1) / kSBufs) & 1u, &s_abort)) {
                             ok = false;
                             break;
                         }
@@ -462,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             s_abort = 1;
             set_status(a.status, kDevTimeout);
         }
-    } else {
+    } else if (warp < 10) {
         // ---------------- output epilogue (warps 6..9) ----------------
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
